@@ -1,0 +1,372 @@
+"""Pins of the fp64 oracle against facts that do not come from the oracle itself.
+
+Each test checks the oracle against brute force, a closed form, an invariant of
+the definitions, hand arithmetic or a number printed in the paper, chosen so
+that a dropped term, a wrong sign or index, or a transposed operand fails one
+of them.  CPU only.
+"""
+import math
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2606_03075_gb300 import synth
+
+RNG = np.random.default_rng(1234)
+
+
+def _rand_case(L=2, H_q=4, H_kv=2, d=8, segments=(("text", 3), ("vision", 5), ("text", 2),
+                                                  ("vision", 4), ("text", 3)),
+               n_win=None, seed=0):
+    rng = np.random.default_rng(seed)
+    modality = np.concatenate([np.full(c, 1 if k == "vision" else 0, np.uint8)
+                               for k, c in segments])
+    text = np.flatnonzero(modality == 0)
+    pos = text if n_win is None else text[-n_win:]
+    n = modality.size
+    q = rng.standard_normal((L, H_q, pos.size, d))
+    k = rng.standard_normal((L, H_kv, n, d))
+    w = rng.random((L, pos.size))
+    w /= w.sum(axis=1, keepdims=True)
+    return q, k, modality, pos.astype(np.int64), w
+
+
+# ---------------------------------------------------------------- P1
+def test_softmax_rows_sum_to_one():
+    q, k, modality, pos, w = _rand_case()
+    for l in range(q.shape[0]):
+        for h in range(q.shape[1]):
+            a = oracle.causal_text_attention(q[l, h], k[l, h // 2], pos, 0.37)
+            assert np.all(np.abs(a.sum(axis=1) - 1.0) < 1e-12)
+            # causal mask: nothing after each row's own position (Eq. 2, M)
+            for i, p in enumerate(pos):
+                assert np.all(a[i, p + 1:] == 0.0)
+                assert np.all(a[i, : p + 1] > 0.0)
+
+
+# ---------------------------------------------------------------- P2
+def test_uniform_attention_closed_form():
+    """Q = 0: every visible key gets 1/(p_i + 1) (Eq. 2), so Eq. 8 and Eq. 5
+    reduce to counting."""
+    q, k, modality, pos, w = _rand_case(L=1, H_q=3, H_kv=3)
+    q[:] = 0.0
+    scores, stat = oracle.twr_scores_tvb_stat(q, k, modality, pos, w, 1.0, 3)
+    vision = np.flatnonzero(modality == 1)
+    expect = np.zeros(vision.size)
+    for vi, j in enumerate(vision):
+        expect[vi] = sum(w[0, i] / (p + 1) for i, p in enumerate(pos) if p >= j)
+    for g in range(3):
+        assert np.allclose(scores[0, g], expect, rtol=1e-13, atol=0)
+    s_expect = 3 * sum(np.count_nonzero(vision <= p) / (p + 1) for p in pos)
+    assert math.isclose(stat[0], s_expect, rel_tol=1e-13)
+
+
+# ---------------------------------------------------------------- P3
+def test_one_hot_saturation():
+    """A query aligned with one key, much larger than the rest, puts all its
+    attention on that key (softmax saturation)."""
+    n, d = 12, 16
+    keys = np.eye(d)[:n]
+    pos = np.array([5, 8, 11])
+    target = np.array([2, 7, 11])
+    q = 80.0 * keys[target]
+    a = oracle.causal_text_attention(q, keys, pos, 1.0)
+    for i, t in enumerate(target):
+        assert a[i, t] > 1.0 - 1e-12
+        others = np.delete(a[i], t)
+        assert np.all(others < 1e-12)
+
+
+# ---------------------------------------------------------------- P4
+def test_mass_consistency_uniform_weights():
+    """With w~ = 1/n_win, summing Eq. 8 over vision keys and heads gives the
+    TV mass of Eq. 5 divided by n_win (and the GQA mean divides by G)."""
+    q, k, modality, pos, _ = _rand_case(L=3, H_q=6, H_kv=2, seed=5)
+    n_win = pos.size
+    w = np.full((3, n_win), 1.0 / n_win)
+    scores, stat = oracle.twr_scores_tvb_stat(q, k, modality, pos, w, 0.5, 2)
+    g = 3
+    for l in range(3):
+        assert math.isclose(g * n_win * scores[l].sum(), stat[l], rel_tol=1e-12)
+        assert 0.0 < stat[l] < 6 * n_win
+
+
+# ---------------------------------------------------------------- P5
+def test_tvb_budget_by_hand():
+    # S = [0.5, 0.3, 0.2], B_V = 7: quotas 3.5, 2.1, 1.4 -> floors 3, 2, 1 and the
+    # single leftover unit goes to the largest fraction (0.5, layer 0).
+    assert oracle.tvb_budgets([0.5, 0.3, 0.2], 7, 100) == [4, 2, 1]
+    # equal fractions: the leftover goes to the lower layer.
+    assert oracle.tvb_budgets([1.0, 1.0, 1.0], 4, 100) == [2, 1, 1]
+    assert oracle.tvb_budgets([1.0, 1.0, 1.0], 5, 100) == [2, 2, 1]
+    # one layer takes everything
+    assert oracle.tvb_budgets([0.37], 11, 100) == [11]
+    # cap: quotas 5.4, 0.3, 0.3 with N_v = 3 -> layer 0 capped at 3; the other
+    # 3 units split 1.5 / 1.5 -> 1 + 1, leftover to the lower layer.
+    assert oracle.tvb_budgets([0.9, 0.05, 0.05], 6, 3) == [3, 2, 1]
+    # zero statistic everywhere: uniform split
+    assert oracle.tvb_budgets([0.0, 0.0, 0.0, 0.0], 6, 10) == [2, 2, 1, 1]
+    # a zero layer gets nothing while others have mass
+    assert oracle.tvb_budgets([0.0, 2.0, 1.0], 6, 10) == [0, 4, 2]
+    # every layer capped
+    assert oracle.tvb_budgets([3.0, 1.0], 8, 4) == [4, 4]
+    with pytest.raises(ValueError):
+        oracle.tvb_budgets([1.0, 1.0], 9, 4)
+
+
+def test_tvb_budget_sums_and_caps_random():
+    rng = np.random.default_rng(7)
+    for _ in range(200):
+        L = int(rng.integers(1, 40))
+        cap = int(rng.integers(1, 50))
+        total = int(rng.integers(0, L * cap + 1))
+        stat = rng.random(L) ** 3
+        b = oracle.tvb_budgets(stat, total, cap)
+        assert sum(b) == total
+        assert all(0 <= x <= cap for x in b)
+        # proportionality: uncapped layers are within one unit of their quota
+        # of what is left after the capped ones
+        capped = [l for l in range(L) if b[l] == cap]
+        free = [l for l in range(L) if l not in capped]
+        rest = total - cap * len(capped)
+        den = sum(stat[l] for l in free)
+        for l in free:
+            assert abs(b[l] - rest * stat[l] / den) < 1.0 + 1e-9
+
+
+def test_vision_budget_totals():
+    # B_V = floor(r * N_v * L + 1/2) for the five workloads
+    cases = {("tiny", 0.25): 16, ("llava15", 0.05): 922, ("llava15", 0.20): 3686,
+             ("next", 0.05): 4608, ("next", 0.10): 9216, ("next", 0.20): 18432,
+             ("qwen25", 0.05): 5734, ("video", 0.05): 11469}
+    for (name, r), expect in cases.items():
+        wl = synth.WORKLOADS[name]
+        assert oracle.vision_budget_total(r, wl.N_v, wl.L) == expect
+
+
+# ---------------------------------------------------------------- P6
+def test_topk_pairwise_definition():
+    """Every kept vision key beats every dropped one: higher score, or the same
+    score at a lower position."""
+    rng = np.random.default_rng(11)
+    modality = (rng.random(60) < 0.7).astype(np.uint8)
+    nv = int(modality.sum())
+    scores = np.round(rng.random((3, 2, nv)) * 8) / 8      # many exact ties
+    budgets = [0, 5, nv]
+    offsets, idx = oracle.tpr_select(scores, budgets, modality)
+    vision = np.flatnonzero(modality == 1)
+    rank = {int(p): r for r, p in enumerate(vision)}
+    for l in range(3):
+        for g in range(2):
+            rows = idx[offsets[l * 2 + g]: offsets[l * 2 + g + 1]]
+            kept = [rank[int(p)] for p in rows if modality[p] == 1]
+            dropped = sorted(set(range(nv)) - set(kept))
+            assert len(kept) == budgets[l]
+            s = scores[l, g]
+            for c in kept:
+                for u in dropped:
+                    assert s[c] > s[u] or (s[c] == s[u] and c < u)
+
+
+def test_topk_all_equal_keeps_lowest_positions():
+    modality = np.array([0, 1, 1, 0, 1, 1, 1, 0], np.uint8)
+    scores = np.ones((1, 1, 5))
+    offsets, idx = oracle.tpr_select(scores, [2], modality)
+    assert idx.tolist() == [0, 1, 2, 3, 7]
+
+
+# ---------------------------------------------------------------- P7
+def test_retained_sets_structure():
+    q, k, modality, pos, w = _rand_case(L=4, H_q=4, H_kv=2, seed=3)
+    scores, stat = oracle.twr_scores_tvb_stat(q, k, modality, pos, w, 0.3, 2)
+    nv = int(modality.sum())
+    total = oracle.vision_budget_total(0.4, nv, 4)
+    budgets = oracle.tvb_budgets(stat, total, nv)
+    offsets, idx = oracle.tpr_select(scores, budgets, modality)
+    text = set(np.flatnonzero(modality == 0).tolist())
+    nt = len(text)
+    assert offsets[0] == 0 and offsets.size == 4 * 2 + 1
+    for l in range(4):
+        for g in range(2):
+            rows = idx[offsets[l * 2 + g]: offsets[l * 2 + g + 1]]
+            assert rows.size == nt + budgets[l]
+            assert text <= set(rows.tolist())
+            assert np.all(np.diff(rows) > 0)
+
+
+# ---------------------------------------------------------------- P8
+def test_table4_memory_arithmetic():
+    """Compacted bytes reproduce the KV memory printed in Table 4 for a
+    LLaVA-1.5-7B-sized cache (all tokens evictable, so the vision basis and the
+    all-token basis coincide)."""
+    path = os.path.join(os.path.dirname(__file__), "golden", "table4_kv_memory.txt")
+    rows = [line.split() for line in open(path) if line.strip() and not line.startswith("#")]
+    L, H_kv, d = 32, 32, 128
+    rng = np.random.default_rng(2)
+    for ctx, ratio, printed in rows:
+        ctx, ratio, printed = int(ctx), float(ratio), float(printed)
+        modality = np.ones(ctx, np.uint8)
+        stat = 0.5 + rng.random(L)
+        total = oracle.vision_budget_total(ratio, ctx, L)
+        budgets = oracle.tvb_budgets(stat, total, ctx)
+        # the per-layer budget is shared by every head of the layer, so one
+        # head per layer is selected and the bytes scaled by H_kv
+        scores = rng.random((L, 1, ctx))
+        offsets, _ = oracle.tpr_select(scores, budgets, modality)
+        gib = H_kv * oracle.compacted_kv_bytes(offsets, d) / 2.0 ** 30
+        assert round(gib, 2) == printed, (ctx, ratio, gib)
+
+
+# ---------------------------------------------------------------- P9
+def test_brute_force_tiny():
+    """Eq. 2, 5, 6, 8 summed term by term with scalar Python loops."""
+    L, H_q, H_kv, d = 2, 4, 2, 5
+    q, k, modality, pos, w = _rand_case(L, H_q, H_kv, d, seed=9)
+    scale = 0.41
+    scores, stat = oracle.twr_scores_tvb_stat(q, k, modality, pos, w, scale, H_kv)
+    G = H_q // H_kv
+    vrank = {}
+    for j, m in enumerate(modality):
+        if m == 1:
+            vrank[j] = len(vrank)
+    bs = np.zeros_like(scores)
+    bstat = np.zeros(L)
+    for l in range(L):
+        for h in range(H_q):
+            g = h // G
+            for i, p in enumerate(pos):
+                logits = []
+                for j in range(p + 1):
+                    dot = 0.0
+                    for c in range(d):
+                        dot += q[l, h, i, c] * k[l, g, j, c]
+                    logits.append(scale * dot)
+                mx = max(logits)
+                e = [math.exp(x - mx) for x in logits]
+                z = sum(e)
+                for j in range(p + 1):
+                    if modality[j] == 1:
+                        a = e[j] / z
+                        bstat[l] += a
+                        bs[l, g, vrank[j]] += w[l, i] * a / G
+    assert np.allclose(scores, bs, rtol=1e-12, atol=1e-15)
+    assert np.allclose(stat, bstat, rtol=1e-12, atol=0)
+
+
+# ---------------------------------------------------------------- more invariants
+def test_gqa_group_mapping_and_mean():
+    """A KV head's score is the mean over its own G query heads h // G == g."""
+    q, k, modality, pos, w = _rand_case(L=2, H_q=6, H_kv=2, seed=21)
+    scores, stat = oracle.twr_scores_tvb_stat(q, k, modality, pos, w, 0.6, 2)
+    for g in range(2):
+        acc = 0.0
+        st = 0.0
+        for h in range(3 * g, 3 * g + 3):
+            s1, t1 = oracle.twr_scores_tvb_stat(q[:, h:h + 1], k[:, g:g + 1], modality, pos,
+                                                w, 0.6, 1)
+            acc = acc + s1[:, 0]
+            st = st + t1
+        assert np.allclose(scores[:, g], acc / 3, rtol=1e-12, atol=1e-16)
+        if g == 0:
+            st0 = st
+    assert np.allclose(stat, st0 + st, rtol=1e-12)
+
+
+def test_key_shift_invariance():
+    """Adding one vector to every key shifts each row's logits by a constant,
+    which the row softmax removes."""
+    q, k, modality, pos, w = _rand_case(seed=4)
+    s0, t0 = oracle.twr_scores_tvb_stat(q, k, modality, pos, w, 0.7, 2)
+    shift = np.random.default_rng(5).standard_normal(k.shape[-1])
+    s1, t1 = oracle.twr_scores_tvb_stat(q, k + shift, modality, pos, w, 0.7, 2)
+    assert np.allclose(s0, s1, rtol=1e-10, atol=1e-14)
+    assert np.allclose(t0, t1, rtol=1e-10)
+
+
+def test_scale_folds_into_queries():
+    q, k, modality, pos, w = _rand_case(seed=6)
+    s0, t0 = oracle.twr_scores_tvb_stat(q, k, modality, pos, w, 0.25, 2)
+    s1, t1 = oracle.twr_scores_tvb_stat(q * 0.25, k, modality, pos, w, 1.0, 2)
+    assert np.allclose(s0, s1, rtol=1e-12, atol=1e-16)
+    assert np.allclose(t0, t1, rtol=1e-12)
+
+
+def test_causality():
+    """Keys after the last query position change nothing; query rows placed
+    before the first vision key carry no text-vision mass."""
+    segs = (("text", 4), ("vision", 6), ("text", 3), ("vision", 5))
+    q, k, modality, pos, w = _rand_case(segments=segs, seed=8)
+    pos = np.array([1, 3, 10, 12])
+    q = q[:, :, :4]
+    w = w[:, :4]
+    s0, t0 = oracle.twr_scores_tvb_stat(q, k, modality, pos, w, 0.5, 2)
+    k2 = k.copy()
+    k2[:, :, 13:] += 3.0
+    s1, t1 = oracle.twr_scores_tvb_stat(q, k2, modality, pos, w, 0.5, 2)
+    assert np.array_equal(s0, s1) and np.array_equal(t0, t1)
+    # the last five vision keys sit after every query row: zero score
+    assert np.all(s0[:, :, 9:] == 0.0)
+    early = np.array([0, 1, 2, 3])
+    _, t_early = oracle.twr_scores_tvb_stat(q, k, modality, early, w, 0.5, 2)
+    assert np.all(t_early == 0.0)
+
+
+def test_linear_in_text_weights():
+    q, k, modality, pos, w = _rand_case(seed=10)
+    w2 = np.random.default_rng(3).random(w.shape)
+    s_a, t_a = oracle.twr_scores_tvb_stat(q, k, modality, pos, w, 0.5, 2)
+    s_b, t_b = oracle.twr_scores_tvb_stat(q, k, modality, pos, w2, 0.5, 2)
+    s_c, t_c = oracle.twr_scores_tvb_stat(q, k, modality, pos, w + 2.0 * w2, 0.5, 2)
+    assert np.allclose(s_c, s_a + 2.0 * s_b, rtol=1e-12, atol=1e-16)
+    assert np.array_equal(t_a, t_b) and np.array_equal(t_a, t_c)
+
+
+def test_widen_bf16_exact():
+    bits = np.array([0x3F80, 0xC000, 0x3F81, 0x0001, 0x7F7F, 0x8000], np.uint16)
+    vals = oracle.widen_bf16(bits)
+    assert vals.tolist() == [1.0, -2.0, 1.0 + 2.0 ** -7, 2.0 ** -133,
+                             (2.0 - 2.0 ** -7) * 2.0 ** 127, -0.0]
+
+
+def test_compact_is_a_row_gather():
+    rng = np.random.default_rng(12)
+    k = rng.integers(-2 ** 15, 2 ** 15, (2, 3, 9, 4), dtype=np.int64).astype(np.int16)
+    v = rng.integers(-2 ** 15, 2 ** 15, (2, 3, 9, 4), dtype=np.int64).astype(np.int16)
+    sets = [[0, 2, 5], [1], [], [3, 4, 8], [0, 1, 2, 3, 4, 5, 6, 7, 8], [7]]
+    offsets = np.cumsum([0] + [len(s) for s in sets])
+    idx = np.array(sum(sets, []), np.int64)
+    ko, vo = oracle.compact(k, v, offsets, idx)
+    r = 0
+    for lg, s in enumerate(sets):
+        l, g = divmod(lg, 3)
+        for p in s:
+            assert np.array_equal(ko[r], k[l, g, p]) and np.array_equal(vo[r], v[l, g, p])
+            r += 1
+    assert r == ko.shape[0]
+
+
+def test_evict_end_to_end_tiny():
+    wl = synth.WORKLOADS["tiny"]
+    inp = synth.generate(wl, seed=0)
+    out = oracle.evict(inp["q"], inp["k"], inp["v"], inp["modality"], inp["text_pos"],
+                       inp["w"], 0.25, wl.H_kv)
+    assert out["budgets"].tolist() == [16]
+    assert out["offsets"][-1] == wl.H_kv * (wl.N_t + 16)
+    # with one layer the statistic is the whole TV mass of 8 heads x 32 rows
+    assert 0.0 < out["stat"][0] < 8 * 32
+
+
+def test_rows_normalised_independently_wide_range():
+    """Rows whose logits differ by ~1000 are each normalised on their own:
+    a row of small logits still sums to one next to a row of huge ones."""
+    n, d = 6, 6
+    keys = np.eye(d)
+    pos = np.array([5, 5])
+    q = np.stack([1000.0 * keys[3], 0.01 * keys[1]])
+    a = oracle.causal_text_attention(q, keys, pos, 1.0)
+    assert np.all(np.isfinite(a))
+    assert np.allclose(a.sum(axis=1), 1.0, rtol=0, atol=1e-12)
+    assert a[0, 3] > 1.0 - 1e-12
+    assert np.all(np.abs(a[1] - 1.0 / 6.0) < 0.01)
