@@ -1,0 +1,167 @@
+/*
+ * tgvkv.h -- C ABI of the TGV-KV eviction step on one GB300 (sm_103a).
+ *
+ * TGV-KV ("Text-Grounded KV Eviction for Vision-Language Models") runs once per
+ * request after the prefill (Section 1; Section 3.3).  Given, for every layer,
+ * the cached keys/values and the queries of the text tokens, it
+ *   1. scores every vision key by text-weighted attention (TWR, Eq. 6-8),
+ *   2. turns each layer's text-vision attention sum into a layer budget
+ *      (TVB, Eq. 5 with x = TV),
+ *   3. keeps all text KV and the top-scoring vision KV of each head
+ *      (TPR, Eq. 10, case b_l > N_t), and
+ *   4. gathers the survivors into a compacted, variable-length cache.
+ * The four steps are the four calls tgvkv_score, tgvkv_budget, tgvkv_select
+ * and tgvkv_compact; tgvkv_evict runs all of them in one call.
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ * - Every data pointer is DEVICE memory on the current CUDA device, owned by
+ *   the caller.  The library never allocates, frees or copies between host and
+ *   device; it never synchronises the stream except in tgvkv_status.
+ * - bf16 tensors are passed as raw 16-bit patterns (uint16_t).
+ * - Every call is asynchronous on `stream` (a cudaStream_t passed as void*;
+ *   NULL = the legacy default stream).
+ * - Arguments are validated on the host before any launch; a bad argument
+ *   returns TGVKV_ERR_INVALID_ARG / TGVKV_ERR_UNSUPPORTED and launches nothing.
+ *   Data-dependent faults found on the device (a query position out of range,
+ *   a modality mask that disagrees with N_v, a budget or index out of range,
+ *   an on-chip wait that gave up) never trap: the kernel skips the bad access
+ *   and sets a bit in the status word inside `workspace`, read back with
+ *   tgvkv_status.
+ * - The message of the last host-side error of the calling thread is returned
+ *   by tgvkv_last_error.
+ * - Pointers to bf16 tensors, `workspace`, and the outputs k_out/v_out must be
+ *   16-byte aligned.
+ *
+ * Budget basis.  The ratio r is the fraction of VISION KV kept over all layers
+ * (the vision-only eviction setting of Appendix B.3, where the TPR policy keeps
+ * every text KV): B_V = floor(r * N_v * L + 1/2) vision rows per head are
+ * shared out over the layers.  Every KV head of layer l keeps the N_t text rows
+ * and b_l vision rows, so the compacted cache holds
+ * H_kv * (L * N_t + B_V) rows (tgvkv_retained_rows).
+ */
+#ifndef TGVKV_H
+#define TGVKV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- return codes ---------------------------------------------------- */
+#define TGVKV_OK              0
+#define TGVKV_ERR_INVALID_ARG 1   /* null / misaligned pointer, bad size or ratio */
+#define TGVKV_ERR_UNSUPPORTED 2   /* a shape this build does not handle (e.g. d) */
+#define TGVKV_ERR_CUDA        3   /* a CUDA runtime call failed (see last_error) */
+#define TGVKV_ERR_DEVICE      4   /* tgvkv_status found device status bits set */
+
+/* ---- device status bits (tgvkv_status) ------------------------------- */
+#define TGVKV_STATUS_TEXT_POS     0x01u /* text_pos not strictly ascending or outside [0, N) */
+#define TGVKV_STATUS_VISION_COUNT 0x02u /* modality marks a vision count other than N_v */
+#define TGVKV_STATUS_BUDGET       0x04u /* a layer budget outside [0, N_v] reached select */
+#define TGVKV_STATUS_INDEX        0x08u /* an index outside [0, N) reached compact */
+#define TGVKV_STATUS_COUNT        0x10u /* a retained set did not hold N_t + b_l rows */
+#define TGVKV_STATUS_TIMEOUT      0x20u /* a bounded on-chip wait gave up */
+
+/* ---- problem description --------------------------------------------- */
+typedef struct tgvkv_desc {
+    int32_t L;              /* decoder layers */
+    int32_t H_q;            /* query heads per layer */
+    int32_t H_kv;           /* KV heads per layer; H_q % H_kv == 0, G = H_q / H_kv */
+    int32_t d;              /* head dimension: 64 or 128 */
+    int32_t N;              /* cached tokens per layer and head (text + vision) */
+    int32_t N_v;            /* vision tokens among them (N_t = N - N_v text tokens) */
+    int32_t n_win;          /* text query rows (positions in text_pos) */
+    float   softmax_scale;  /* logits = softmax_scale * <q, k>; <= 0 means 1/sqrt(d) */
+    int64_t w_layer_stride; /* floats between the weight rows of two layers; 0 = one
+                               row shared by every layer */
+} tgvkv_desc;
+
+/* Bytes of device workspace the calls below need for this problem. */
+size_t tgvkv_workspace_size(const tgvkv_desc* desc);
+
+/* B_V = floor(ratio * N_v * L + 1/2): vision rows kept per KV head over all
+ * layers (Eq. 5 splits it).  Returns -1 if desc or ratio (not in [0,1]) is bad. */
+int64_t tgvkv_vision_budget_total(const tgvkv_desc* desc, double ratio);
+
+/* Rows of the compacted cache, H_kv * (L * N_t + B_V); the capacity that idx,
+ * k_out and v_out must have.  Returns -1 on bad arguments. */
+int64_t tgvkv_retained_rows(const tgvkv_desc* desc, double ratio);
+
+/* TWR scores and the TVB statistic (Eq. 2, 5, 6, 8).
+ *
+ * For every layer l and query head h (KV head g = h / G), every query row i at
+ * sequence position text_pos[i] attends causally to the keys 0..text_pos[i]
+ * with A = softmax(softmax_scale * q k^T) over ALL of those keys (Eq. 2); the
+ * text-vision attention is the slice of A on vision keys (Eq. 6).
+ *   scores[l][g][v] = (1/G) sum_{h in g} sum_i w[l][i] * A_{l,h}[i, v]   (Eq. 8)
+ *   tvb_stat[l]     = sum_h sum_i sum_v A_{l,h}[i, v]       (Eq. 5 numerator)
+ * where v = 0..N_v-1 runs over the vision keys in position order.
+ *
+ * q_text:   bf16 [L][H_q][n_win][d]
+ * k:        bf16 [L][H_kv][N][d]          (the key cache)
+ * modality: uint8 [N], 1 = vision token, 0 = text token (same for all layers)
+ * text_pos: int32 [n_win], strictly ascending positions in [0, N)
+ * w:        fp32 text weights w~, row l at w + l * w_layer_stride, n_win floats
+ * scores:   fp32 [L][H_kv][N_v]  (output)
+ * tvb_stat: fp32 [L]             (output)
+ * Arithmetic: bf16 products, fp32 accumulation and fp32 softmax. */
+int tgvkv_score(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* k,
+                const uint8_t* modality, const int32_t* text_pos, const float* w,
+                float* scores, float* tvb_stat, void* workspace, void* stream);
+
+/* TVB layer budgets (Eq. 5, x = TV).  Splits B_V over the layers in proportion
+ * to tvb_stat: b_l = floor(B_V * S_l / sum S) plus one leftover unit each for
+ * the largest fractional parts (ties: lower layer); a layer above N_v is capped
+ * at N_v and the rest re-split over the other layers; all-zero statistics give a
+ * uniform split.  The quotients are computed in double on the device.
+ * tvb_stat: fp32 [L]; budgets: int32 [L] (output, vision rows per KV head). */
+int tgvkv_budget(const tgvkv_desc* desc, const float* tvb_stat, double ratio,
+                 int32_t* budgets, void* workspace, void* stream);
+
+/* TPR retention (Eq. 10, case b_l > N_t with the vision budget b_l).
+ * For every (l, g): every text position plus the budgets[l] vision positions
+ * with the largest scores[l][g][.] (ties: lower position), in ascending
+ * position order.  The sets are stored as CSR over (l, g) in row-major order:
+ * set (l, g) is idx[offsets[l*H_kv+g] .. offsets[l*H_kv+g+1]).
+ * offsets: int64 [L*H_kv + 1] (output); idx: int32 positions (output, capacity
+ * tgvkv_retained_rows). */
+int tgvkv_select(const tgvkv_desc* desc, const float* scores, const int32_t* budgets,
+                 const uint8_t* modality, int64_t* offsets, int32_t* idx,
+                 void* workspace, void* stream);
+
+/* Compaction: row r of set (l, g) of the CSR becomes
+ *   k_out[r] = k[l][g][idx[r]],  v_out[r] = v[l][g][idx[r]]
+ * as bit copies.  k, v: bf16 [L][H_kv][N][d]; k_out, v_out: bf16
+ * [offsets[L*H_kv]][d] (output; capacity tgvkv_retained_rows rows). */
+int tgvkv_compact(const tgvkv_desc* desc, const uint16_t* k, const uint16_t* v,
+                  const int64_t* offsets, const int32_t* idx,
+                  uint16_t* k_out, uint16_t* v_out, void* workspace, void* stream);
+
+/* score -> budget -> select -> compact in one stream-ordered call with no host
+ * synchronisation.  Arguments as in the four calls above. */
+int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* k,
+                const uint16_t* v, const uint8_t* modality, const int32_t* text_pos,
+                const float* w, double ratio,
+                float* scores, float* tvb_stat, int32_t* budgets,
+                int64_t* offsets, int32_t* idx, uint16_t* k_out, uint16_t* v_out,
+                void* workspace, void* stream);
+
+/* Zero `workspace` (asynchronously on `stream`).  Needed once after the
+ * workspace is allocated; the calls keep it consistent afterwards. */
+int tgvkv_workspace_init(const tgvkv_desc* desc, void* workspace, void* stream);
+
+/* Synchronise `stream`, then read and clear the device status word kept in
+ * `workspace`.  Returns the TGVKV_STATUS_* bits (0 = clean) or a negative
+ * value if the synchronisation itself failed. */
+int tgvkv_status(void* workspace, void* stream);
+
+/* Message of the last error returned on the calling thread ("" if none). */
+const char* tgvkv_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* TGVKV_H */

@@ -1,0 +1,214 @@
+"""Python binding of the TGV-KV C ABI (include/tgvkv.h).
+
+Argument marshalling only: each function checks that the torch tensors have
+the dtype, device, contiguity and size the C call expects, passes their device
+pointers and the current CUDA stream, and raises on a non-zero return code.
+Every step of the computation runs in the library's CUDA kernels.  PyTorch
+provides device memory and streams.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+from dataclasses import dataclass
+
+import torch
+
+from . import _lib
+
+Desc = _lib.Desc
+
+_BF16_LIKE = (torch.bfloat16, torch.int16, torch.uint16)
+
+
+class TgvkvError(RuntimeError):
+    def __init__(self, code, fn):
+        msg = _lib.load().tgvkv_last_error().decode()
+        super().__init__(f"{fn} failed with code {code}: {msg}")
+        self.code = code
+
+
+def make_desc(L, H_q, H_kv, d, N, N_v, n_win, softmax_scale=0.0, w_layer_stride=None) -> Desc:
+    """A problem descriptor; w_layer_stride defaults to n_win (one weight row per layer)."""
+    return Desc(L=L, H_q=H_q, H_kv=H_kv, d=d, N=N, N_v=N_v, n_win=n_win,
+                softmax_scale=float(softmax_scale),
+                w_layer_stride=n_win if w_layer_stride is None else w_layer_stride)
+
+
+def desc_for_workload(wl, softmax_scale=0.0) -> Desc:
+    return make_desc(wl.L, wl.H_q, wl.H_kv, wl.d, wl.N, wl.N_v, wl.n_win, softmax_scale)
+
+
+def _stream(stream):
+    if stream is None:
+        return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, torch.cuda.Stream):
+        return ctypes.c_void_p(stream.cuda_stream)
+    return ctypes.c_void_p(int(stream))
+
+
+def _ptr(t, dtypes, numel, name):
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if t.dtype not in dtypes:
+        raise TypeError(f"{name} has dtype {t.dtype}, expected one of {dtypes}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if t.numel() < numel:
+        raise ValueError(f"{name} holds {t.numel()} elements, needs {numel}")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _check(code, fn):
+    if code != 0:
+        raise TgvkvError(code, fn)
+
+
+def tgvkv_workspace_size(desc: Desc) -> int:
+    n = _lib.load().tgvkv_workspace_size(ctypes.byref(desc))
+    if n == 0:
+        raise TgvkvError(-1, "tgvkv_workspace_size")
+    return int(n)
+
+
+def tgvkv_vision_budget_total(desc: Desc, ratio: float) -> int:
+    n = _lib.load().tgvkv_vision_budget_total(ctypes.byref(desc), float(ratio))
+    if n < 0:
+        raise TgvkvError(-1, "tgvkv_vision_budget_total")
+    return int(n)
+
+
+def tgvkv_retained_rows(desc: Desc, ratio: float) -> int:
+    n = _lib.load().tgvkv_retained_rows(ctypes.byref(desc), float(ratio))
+    if n < 0:
+        raise TgvkvError(-1, "tgvkv_retained_rows")
+    return int(n)
+
+
+def tgvkv_workspace_init(desc: Desc, ws: torch.Tensor, stream=None):
+    p = _ptr(ws, (torch.uint8,), tgvkv_workspace_size(desc), "workspace")
+    _check(_lib.load().tgvkv_workspace_init(ctypes.byref(desc), p, _stream(stream)),
+           "tgvkv_workspace_init")
+
+
+def new_workspace(desc: Desc, device=None) -> torch.Tensor:
+    """A zeroed workspace tensor (uint8) for this problem."""
+    ws = torch.empty(tgvkv_workspace_size(desc), dtype=torch.uint8, device=device or "cuda")
+    tgvkv_workspace_init(desc, ws)
+    return ws
+
+
+def tgvkv_score(desc, q_text, k, modality, text_pos, w, scores, tvb_stat, ws, stream=None):
+    L, Hq, Hkv, d, N, Nv, nw = desc.L, desc.H_q, desc.H_kv, desc.d, desc.N, desc.N_v, desc.n_win
+    wrows = (L - 1) * desc.w_layer_stride + nw if nw else 0
+    _check(_lib.load().tgvkv_score(
+        ctypes.byref(desc),
+        _ptr(q_text, _BF16_LIKE, L * Hq * nw * d, "q_text"),
+        _ptr(k, _BF16_LIKE, L * Hkv * N * d, "k"),
+        _ptr(modality, (torch.uint8,), N, "modality"),
+        _ptr(text_pos, (torch.int32,), nw, "text_pos"),
+        _ptr(w, (torch.float32,), wrows, "w"),
+        _ptr(scores, (torch.float32,), L * Hkv * Nv, "scores"),
+        _ptr(tvb_stat, (torch.float32,), L, "tvb_stat"),
+        _ptr(ws, (torch.uint8,), tgvkv_workspace_size(desc), "workspace"),
+        _stream(stream)), "tgvkv_score")
+
+
+def tgvkv_budget(desc, tvb_stat, ratio, budgets, ws, stream=None):
+    _check(_lib.load().tgvkv_budget(
+        ctypes.byref(desc),
+        _ptr(tvb_stat, (torch.float32,), desc.L, "tvb_stat"), float(ratio),
+        _ptr(budgets, (torch.int32,), desc.L, "budgets"),
+        _ptr(ws, (torch.uint8,), tgvkv_workspace_size(desc), "workspace"),
+        _stream(stream)), "tgvkv_budget")
+
+
+def tgvkv_select(desc, scores, budgets, modality, offsets, idx, ws, stream=None):
+    LH = desc.L * desc.H_kv
+    _check(_lib.load().tgvkv_select(
+        ctypes.byref(desc),
+        _ptr(scores, (torch.float32,), LH * desc.N_v, "scores"),
+        _ptr(budgets, (torch.int32,), desc.L, "budgets"),
+        _ptr(modality, (torch.uint8,), desc.N, "modality"),
+        _ptr(offsets, (torch.int64,), LH + 1, "offsets"),
+        _ptr(idx, (torch.int32,), 0, "idx"),
+        _ptr(ws, (torch.uint8,), tgvkv_workspace_size(desc), "workspace"),
+        _stream(stream)), "tgvkv_select")
+
+
+def tgvkv_compact(desc, k, v, offsets, idx, k_out, v_out, ws, stream=None):
+    n = desc.L * desc.H_kv * desc.N * desc.d
+    _check(_lib.load().tgvkv_compact(
+        ctypes.byref(desc),
+        _ptr(k, _BF16_LIKE, n, "k"), _ptr(v, _BF16_LIKE, n, "v"),
+        _ptr(offsets, (torch.int64,), desc.L * desc.H_kv + 1, "offsets"),
+        _ptr(idx, (torch.int32,), 0, "idx"),
+        _ptr(k_out, _BF16_LIKE, 0, "k_out"), _ptr(v_out, _BF16_LIKE, 0, "v_out"),
+        _ptr(ws, (torch.uint8,), tgvkv_workspace_size(desc), "workspace"),
+        _stream(stream)), "tgvkv_compact")
+
+
+@dataclass
+class EvictOutputs:
+    scores: torch.Tensor     # fp32 [L, H_kv, N_v]
+    tvb_stat: torch.Tensor   # fp32 [L]
+    budgets: torch.Tensor    # int32 [L]
+    offsets: torch.Tensor    # int64 [L*H_kv + 1]
+    idx: torch.Tensor        # int32 [retained rows]
+    k_out: torch.Tensor      # bf16 [retained rows, d]
+    v_out: torch.Tensor      # bf16 [retained rows, d]
+
+
+def alloc_outputs(desc: Desc, ratio: float, device=None) -> EvictOutputs:
+    dev = device or "cuda"
+    rows = tgvkv_retained_rows(desc, ratio)
+    L, Hkv = desc.L, desc.H_kv
+    return EvictOutputs(
+        scores=torch.empty((L, Hkv, desc.N_v), dtype=torch.float32, device=dev),
+        tvb_stat=torch.empty(L, dtype=torch.float32, device=dev),
+        budgets=torch.empty(L, dtype=torch.int32, device=dev),
+        offsets=torch.empty(L * Hkv + 1, dtype=torch.int64, device=dev),
+        idx=torch.empty(max(rows, 1), dtype=torch.int32, device=dev),
+        k_out=torch.empty((max(rows, 1), desc.d), dtype=torch.bfloat16, device=dev),
+        v_out=torch.empty((max(rows, 1), desc.d), dtype=torch.bfloat16, device=dev))
+
+
+def tgvkv_evict(desc, q_text, k, v, modality, text_pos, w, ratio, out: EvictOutputs, ws,
+                stream=None):
+    L, Hq, Hkv, d, N, Nv, nw = desc.L, desc.H_q, desc.H_kv, desc.d, desc.N, desc.N_v, desc.n_win
+    rows = tgvkv_retained_rows(desc, ratio)
+    wrows = (L - 1) * desc.w_layer_stride + nw if nw else 0
+    _check(_lib.load().tgvkv_evict(
+        ctypes.byref(desc),
+        _ptr(q_text, _BF16_LIKE, L * Hq * nw * d, "q_text"),
+        _ptr(k, _BF16_LIKE, L * Hkv * N * d, "k"),
+        _ptr(v, _BF16_LIKE, L * Hkv * N * d, "v"),
+        _ptr(modality, (torch.uint8,), N, "modality"),
+        _ptr(text_pos, (torch.int32,), nw, "text_pos"),
+        _ptr(w, (torch.float32,), wrows, "w"),
+        float(ratio),
+        _ptr(out.scores, (torch.float32,), L * Hkv * Nv, "scores"),
+        _ptr(out.tvb_stat, (torch.float32,), L, "tvb_stat"),
+        _ptr(out.budgets, (torch.int32,), L, "budgets"),
+        _ptr(out.offsets, (torch.int64,), L * Hkv + 1, "offsets"),
+        _ptr(out.idx, (torch.int32,), rows, "idx"),
+        _ptr(out.k_out, _BF16_LIKE, rows * d, "k_out"),
+        _ptr(out.v_out, _BF16_LIKE, rows * d, "v_out"),
+        _ptr(ws, (torch.uint8,), tgvkv_workspace_size(desc), "workspace"),
+        _stream(stream)), "tgvkv_evict")
+
+
+def tgvkv_status(ws: torch.Tensor, stream=None) -> int:
+    """Synchronise the stream, return and clear the device status bits."""
+    rc = _lib.load().tgvkv_status(_ptr(ws, (torch.uint8,), 4, "workspace"), _stream(stream))
+    if rc < 0:
+        raise TgvkvError(-rc, "tgvkv_status")
+    return rc
+
+
+def default_scale(d: int) -> float:
+    return 1.0 / math.sqrt(d)

@@ -1,0 +1,296 @@
+// C ABI of the TGV-KV eviction step: argument checks on the host, workspace
+// layout, and the stream-ordered launches of the four kernels.
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include "common.cuh"
+#include "launch.h"
+#include "tgvkv.h"
+
+namespace tgvkv {
+namespace {
+
+thread_local char g_last_error[512] = "";
+
+int fail(int code, const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_last_error, sizeof(g_last_error), fmt, ap);
+    va_end(ap);
+    return code;
+}
+
+int ok() {
+    g_last_error[0] = '\0';
+    return TGVKV_OK;
+}
+
+int cuda_fail(cudaError_t e, const char* what) {
+    return fail(TGVKV_ERR_CUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+bool aligned16(const void* ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; }
+
+size_t round_up(size_t x) { return (x + 255) & ~size_t(255); }
+
+WsLayout layout_of(const Problem& p) {
+    WsLayout w;
+    size_t o = 0;
+    w.status = o;      o += round_up(sizeof(uint32_t));
+    w.tickets = o;     o += round_up(sizeof(uint32_t) * (size_t)(p.L * p.H_kv + p.L));
+    w.stat_part = o;   o += round_up(sizeof(float) * (size_t)p.L * p.H_kv * (p.T > 0 ? p.T : 1));
+    w.stat_head = o;   o += round_up(sizeof(float) * (size_t)p.L * p.H_kv);
+    w.score_part = o;
+    if (p.T > 1) o += round_up(sizeof(float) * (size_t)p.L * p.H_kv * p.T * (size_t)p.N_v);
+    w.total = o;
+    return w;
+}
+
+// Validate a descriptor and build the kernels' view of it.
+int make_problem(const tgvkv_desc* d, Problem* p) {
+    if (!d) return fail(TGVKV_ERR_INVALID_ARG, "desc is NULL");
+    if (d->L < 1 || d->H_q < 1 || d->H_kv < 1 || d->N < 1 || d->n_win < 0 || d->N_v < 0 ||
+        d->N_v > d->N)
+        return fail(TGVKV_ERR_INVALID_ARG,
+                    "bad sizes: L=%d H_q=%d H_kv=%d N=%d N_v=%d n_win=%d", d->L, d->H_q, d->H_kv,
+                    d->N, d->N_v, d->n_win);
+    if (d->H_q % d->H_kv != 0)
+        return fail(TGVKV_ERR_INVALID_ARG, "H_q=%d is not a multiple of H_kv=%d", d->H_q, d->H_kv);
+    if (d->d != 64 && d->d != 128)
+        return fail(TGVKV_ERR_UNSUPPORTED, "head dim %d unsupported (64 or 128)", d->d);
+    if (d->N > kMaxN) return fail(TGVKV_ERR_UNSUPPORTED, "N=%d above %d", d->N, kMaxN);
+    if (d->N_v > kMaxNv) return fail(TGVKV_ERR_UNSUPPORTED, "N_v=%d above %d", d->N_v, kMaxNv);
+    if (d->L > kMaxL) return fail(TGVKV_ERR_UNSUPPORTED, "L=%d above %d", d->L, kMaxL);
+    if (d->w_layer_stride < 0)
+        return fail(TGVKV_ERR_INVALID_ARG, "w_layer_stride=%lld < 0", (long long)d->w_layer_stride);
+    if (!(d->softmax_scale == d->softmax_scale) || isinf(d->softmax_scale))
+        return fail(TGVKV_ERR_INVALID_ARG, "softmax_scale is not finite");
+    const long long rows = (long long)(d->H_q / d->H_kv) * d->n_win;
+    if (rows > (1LL << 24)) return fail(TGVKV_ERR_UNSUPPORTED, "G * n_win = %lld too large", rows);
+    if ((long long)d->L * d->H_kv > 65535)
+        return fail(TGVKV_ERR_UNSUPPORTED, "L * H_kv above 65535");
+    p->L = d->L;
+    p->H_q = d->H_q;
+    p->H_kv = d->H_kv;
+    p->G = d->H_q / d->H_kv;
+    p->d = d->d;
+    p->N = d->N;
+    p->N_v = d->N_v;
+    p->N_t = d->N - d->N_v;
+    p->n_win = d->n_win;
+    p->R = (int)rows;
+    p->T = (p->R + 127) / 128;
+    const double scale = d->softmax_scale > 0.f ? (double)d->softmax_scale : 1.0 / sqrt((double)d->d);
+    p->scale_log2 = (float)(scale * 1.4426950408889634);  // log2(e)
+    p->w_stride = (long long)d->w_layer_stride;
+    return TGVKV_OK;
+}
+
+int check_ratio(double ratio) {
+    if (!(ratio >= 0.0 && ratio <= 1.0))
+        return fail(TGVKV_ERR_INVALID_ARG, "ratio %g outside [0, 1]", ratio);
+    return TGVKV_OK;
+}
+
+long long budget_total(const Problem& p, double ratio) {
+    return (long long)floor(ratio * (double)((long long)p.N_v * p.L) + 0.5);
+}
+
+long long retained_rows(const Problem& p, double ratio) {
+    return (long long)p.H_kv * ((long long)p.L * p.N_t + budget_total(p, ratio));
+}
+
+#define REQUIRE_PTR(ptr, name, need16)                                                   \
+    do {                                                                                 \
+        if (!(ptr)) return fail(TGVKV_ERR_INVALID_ARG, "%s is NULL", name);              \
+        if ((need16) && !aligned16(ptr))                                                 \
+            return fail(TGVKV_ERR_INVALID_ARG, "%s is not 16-byte aligned", name);       \
+    } while (0)
+
+uint32_t* status_of(void* ws, const WsLayout& lay) {
+    return reinterpret_cast<uint32_t*>(static_cast<char*>(ws) + lay.status);
+}
+
+int do_score(const Problem& p, const uint16_t* q, const uint16_t* k, const uint8_t* modality,
+             const int32_t* text_pos, const float* w, float* scores, float* tvb_stat, void* ws,
+             cudaStream_t st) {
+    const WsLayout lay = layout_of(p);
+    cudaError_t e = launch_score(p, q, k, modality, text_pos, w, scores, tvb_stat,
+                                 static_cast<char*>(ws), lay, st);
+    return e == cudaSuccess ? TGVKV_OK : cuda_fail(e, "score launch");
+}
+
+int check_score_args(const Problem& p, const uint16_t* q, const uint16_t* k,
+                     const uint8_t* modality, const int32_t* text_pos, const float* w,
+                     const float* scores, const float* tvb_stat, const void* ws) {
+    if (p.n_win > 0) {
+        REQUIRE_PTR(q, "q_text", true);
+        REQUIRE_PTR(text_pos, "text_pos", false);
+        REQUIRE_PTR(w, "w", false);
+    }
+    REQUIRE_PTR(k, "k", true);
+    REQUIRE_PTR(modality, "modality", false);
+    if (p.N_v > 0) REQUIRE_PTR(scores, "scores", false);
+    REQUIRE_PTR(tvb_stat, "tvb_stat", false);
+    REQUIRE_PTR(ws, "workspace", true);
+    return TGVKV_OK;
+}
+
+}  // namespace
+}  // namespace tgvkv
+
+using namespace tgvkv;
+
+extern "C" {
+
+size_t tgvkv_workspace_size(const tgvkv_desc* desc) {
+    Problem p{};
+    if (make_problem(desc, &p) != TGVKV_OK) return 0;
+    return layout_of(p).total;
+}
+
+int64_t tgvkv_vision_budget_total(const tgvkv_desc* desc, double ratio) {
+    Problem p{};
+    if (make_problem(desc, &p) != TGVKV_OK || check_ratio(ratio) != TGVKV_OK) return -1;
+    return budget_total(p, ratio);
+}
+
+int64_t tgvkv_retained_rows(const tgvkv_desc* desc, double ratio) {
+    Problem p{};
+    if (make_problem(desc, &p) != TGVKV_OK || check_ratio(ratio) != TGVKV_OK) return -1;
+    return retained_rows(p, ratio);
+}
+
+int tgvkv_score(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* k,
+                const uint8_t* modality, const int32_t* text_pos, const float* w,
+                float* scores, float* tvb_stat, void* workspace, void* stream) {
+    Problem p{};
+    int rc = make_problem(desc, &p);
+    if (rc) return rc;
+    rc = check_score_args(p, q_text, k, modality, text_pos, w, scores, tvb_stat, workspace);
+    if (rc) return rc;
+    rc = do_score(p, q_text, k, modality, text_pos, w, scores, tvb_stat, workspace,
+                  static_cast<cudaStream_t>(stream));
+    return rc ? rc : ok();
+}
+
+int tgvkv_budget(const tgvkv_desc* desc, const float* tvb_stat, double ratio, int32_t* budgets,
+                 void* workspace, void* stream) {
+    Problem p{};
+    int rc = make_problem(desc, &p);
+    if (rc) return rc;
+    if ((rc = check_ratio(ratio))) return rc;
+    REQUIRE_PTR(tvb_stat, "tvb_stat", false);
+    REQUIRE_PTR(budgets, "budgets", false);
+    REQUIRE_PTR(workspace, "workspace", true);
+    const WsLayout lay = layout_of(p);
+    cudaError_t e = launch_budget(p, tvb_stat, budget_total(p, ratio), budgets,
+                                  status_of(workspace, lay), static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ok() : cuda_fail(e, "budget launch");
+}
+
+int tgvkv_select(const tgvkv_desc* desc, const float* scores, const int32_t* budgets,
+                 const uint8_t* modality, int64_t* offsets, int32_t* idx, void* workspace,
+                 void* stream) {
+    Problem p{};
+    int rc = make_problem(desc, &p);
+    if (rc) return rc;
+    if (p.N_v > 0) REQUIRE_PTR(scores, "scores", false);
+    REQUIRE_PTR(budgets, "budgets", false);
+    REQUIRE_PTR(modality, "modality", false);
+    REQUIRE_PTR(offsets, "offsets", false);
+    REQUIRE_PTR(idx, "idx", false);
+    REQUIRE_PTR(workspace, "workspace", true);
+    const WsLayout lay = layout_of(p);
+    cudaError_t e = launch_select(p, scores, budgets, modality, offsets, idx,
+                                  status_of(workspace, lay), static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ok() : cuda_fail(e, "select launch");
+}
+
+int tgvkv_compact(const tgvkv_desc* desc, const uint16_t* k, const uint16_t* v,
+                  const int64_t* offsets, const int32_t* idx, uint16_t* k_out, uint16_t* v_out,
+                  void* workspace, void* stream) {
+    Problem p{};
+    int rc = make_problem(desc, &p);
+    if (rc) return rc;
+    REQUIRE_PTR(k, "k", true);
+    REQUIRE_PTR(v, "v", true);
+    REQUIRE_PTR(offsets, "offsets", false);
+    REQUIRE_PTR(idx, "idx", false);
+    REQUIRE_PTR(k_out, "k_out", true);
+    REQUIRE_PTR(v_out, "v_out", true);
+    REQUIRE_PTR(workspace, "workspace", true);
+    const WsLayout lay = layout_of(p);
+    // every set holds at most N rows
+    const long long cap = (long long)p.L * p.H_kv * p.N;
+    cudaError_t e = launch_compact(p, k, v, offsets, idx, k_out, v_out, cap,
+                                   status_of(workspace, lay), static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ok() : cuda_fail(e, "compact launch");
+}
+
+int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* k,
+                const uint16_t* v, const uint8_t* modality, const int32_t* text_pos,
+                const float* w, double ratio, float* scores, float* tvb_stat, int32_t* budgets,
+                int64_t* offsets, int32_t* idx, uint16_t* k_out, uint16_t* v_out,
+                void* workspace, void* stream) {
+    Problem p{};
+    int rc = make_problem(desc, &p);
+    if (rc) return rc;
+    if ((rc = check_ratio(ratio))) return rc;
+    rc = check_score_args(p, q_text, k, modality, text_pos, w, scores, tvb_stat, workspace);
+    if (rc) return rc;
+    REQUIRE_PTR(v, "v", true);
+    REQUIRE_PTR(budgets, "budgets", false);
+    REQUIRE_PTR(offsets, "offsets", false);
+    REQUIRE_PTR(idx, "idx", false);
+    REQUIRE_PTR(k_out, "k_out", true);
+    REQUIRE_PTR(v_out, "v_out", true);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const WsLayout lay = layout_of(p);
+    uint32_t* status = status_of(workspace, lay);
+    cudaError_t e = launch_score(p, q_text, k, modality, text_pos, w, scores, tvb_stat,
+                                 static_cast<char*>(workspace), lay, st);
+    if (e != cudaSuccess) return cuda_fail(e, "score launch");
+    e = launch_budget(p, tvb_stat, budget_total(p, ratio), budgets, status, st);
+    if (e != cudaSuccess) return cuda_fail(e, "budget launch");
+    e = launch_select(p, scores, budgets, modality, offsets, idx, status, st);
+    if (e != cudaSuccess) return cuda_fail(e, "select launch");
+    e = launch_compact(p, k, v, offsets, idx, k_out, v_out, retained_rows(p, ratio), status, st);
+    if (e != cudaSuccess) return cuda_fail(e, "compact launch");
+    return ok();
+}
+
+int tgvkv_workspace_init(const tgvkv_desc* desc, void* workspace, void* stream) {
+    Problem p{};
+    int rc = make_problem(desc, &p);
+    if (rc) return rc;
+    REQUIRE_PTR(workspace, "workspace", true);
+    cudaError_t e = cudaMemsetAsync(workspace, 0, layout_of(p).total, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ok() : cuda_fail(e, "workspace memset");
+}
+
+int tgvkv_status(void* workspace, void* stream) {
+    if (!workspace) {
+        fail(TGVKV_ERR_INVALID_ARG, "workspace is NULL");
+        return -TGVKV_ERR_INVALID_ARG;
+    }
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    uint32_t bits = 0;
+    // the status word sits at offset 0 of every workspace layout
+    cudaError_t e = cudaStreamSynchronize(st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&bits, workspace, sizeof(bits), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(workspace, 0, sizeof(bits), st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) {
+        cuda_fail(e, "status read");
+        return -TGVKV_ERR_CUDA;
+    }
+    ok();
+    return (int)bits;
+}
+
+const char* tgvkv_last_error(void) { return g_last_error; }
+
+}  // extern "C"

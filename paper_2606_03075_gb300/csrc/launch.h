@@ -1,0 +1,30 @@
+// Host-side launchers of the TGV-KV kernels (one per step).  All of them are
+// asynchronous on `stream` and assume the arguments were validated by the
+// C-ABI layer.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "common.cuh"
+
+namespace tgvkv {
+
+cudaError_t launch_score(const Problem& p, const uint16_t* q, const uint16_t* k,
+                         const uint8_t* modality, const int32_t* text_pos, const float* w,
+                         float* scores, float* tvb_stat, char* ws, const WsLayout& lay,
+                         cudaStream_t stream);
+
+cudaError_t launch_budget(const Problem& p, const float* tvb_stat, long long total,
+                          int32_t* budgets, uint32_t* status, cudaStream_t stream);
+
+cudaError_t launch_select(const Problem& p, const float* scores, const int32_t* budgets,
+                          const uint8_t* modality, int64_t* offsets, int32_t* idx,
+                          uint32_t* status, cudaStream_t stream);
+
+cudaError_t launch_compact(const Problem& p, const uint16_t* k, const uint16_t* v,
+                           const int64_t* offsets, const int32_t* idx, uint16_t* k_out,
+                           uint16_t* v_out, long long capacity_rows, uint32_t* status,
+                           cudaStream_t stream);
+
+}  // namespace tgvkv

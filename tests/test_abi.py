@@ -1,0 +1,93 @@
+"""C-ABI surface checks that need no GPU: the library builds and loads, every
+function declared in include/tgvkv.h is exported, host-side validation rejects
+bad arguments before any launch, and the host-side budget arithmetic agrees
+with the oracle."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2606_03075_gb300 import synth
+
+
+@pytest.fixture(scope="module")
+def lib(repo_root):
+    from paper_2606_03075_gb300 import build
+    build.build()
+    from paper_2606_03075_gb300 import _lib
+    return _lib.load()
+
+
+def _declared(repo_root):
+    src = open(os.path.join(repo_root, "include", "tgvkv.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(tgvkv_[a-z_]+)\s*\(", src)))
+
+
+def test_exports_every_declared_symbol(lib, repo_root):
+    from paper_2606_03075_gb300 import _lib
+    names = _declared(repo_root)
+    assert len(names) >= 11
+    for name in names:
+        assert hasattr(lib, name), name
+    assert sorted(_lib.SIGNATURES) == names
+
+
+def _desc(**kw):
+    from paper_2606_03075_gb300 import _lib
+    base = dict(L=2, H_q=4, H_kv=2, d=128, N=100, N_v=60, n_win=8, softmax_scale=0.0,
+                w_layer_stride=8)
+    base.update(kw)
+    return _lib.Desc(**base)
+
+
+def test_validation_rejects_before_launch(lib):
+    P = ctypes.c_void_p
+    fake = P(0x1000)        # never dereferenced: every call below fails validation
+    odd = P(0x1008)         # 8-byte aligned only
+    d = _desc()
+    ref = ctypes.byref
+
+    def score(desc, q=fake, k=fake, ws=fake):
+        return lib.tgvkv_score(desc, q, k, fake, fake, fake, fake, fake, ws, None)
+
+    assert score(None) == 1
+    assert score(ref(_desc(d=96))) == 2
+    assert score(ref(_desc(H_q=3))) == 1
+    assert score(ref(_desc(N_v=101))) == 1
+    assert score(ref(_desc(N=70000, N_v=10))) == 2
+    assert score(ref(d), q=P(0)) == 1
+    assert score(ref(d), k=odd) == 1
+    assert score(ref(d), ws=odd) == 1
+    assert b"16-byte" in lib.tgvkv_last_error()
+    assert lib.tgvkv_budget(ref(d), fake, 1.5, fake, fake, None) == 1
+    assert lib.tgvkv_budget(ref(d), fake, -0.1, fake, fake, None) == 1
+    assert lib.tgvkv_budget(ref(d), fake, float("nan"), fake, fake, None) == 1
+    assert lib.tgvkv_select(ref(d), fake, fake, fake, fake, P(0), fake, None) == 1
+    assert lib.tgvkv_compact(ref(d), fake, fake, fake, fake, odd, fake, fake, None) == 1
+    assert lib.tgvkv_evict(ref(d), fake, fake, fake, fake, fake, fake, 2.0, fake, fake, fake,
+                           fake, fake, fake, fake, fake, None) == 1
+    assert lib.tgvkv_workspace_size(ref(_desc(d=32))) == 0
+    assert lib.tgvkv_retained_rows(ref(d), 1.01) == -1
+    assert lib.tgvkv_status(None, None) < 0
+
+
+def test_host_budget_arithmetic_matches_oracle(lib):
+    ref = ctypes.byref
+    for name, wl in synth.WORKLOADS.items():
+        d = _desc(L=wl.L, H_q=wl.H_q, H_kv=wl.H_kv, d=wl.d, N=wl.N, N_v=wl.N_v, n_win=wl.n_win,
+                  w_layer_stride=wl.n_win)
+        for r in (0.0, 0.05, 0.1, 0.2, 0.25, 0.5, 1.0) + tuple(wl.ratios):
+            bv = oracle.vision_budget_total(r, wl.N_v, wl.L)
+            assert lib.tgvkv_vision_budget_total(ref(d), r) == bv
+            assert lib.tgvkv_retained_rows(ref(d), r) == wl.H_kv * (wl.L * wl.N_t + bv)
+        assert lib.tgvkv_workspace_size(ref(d)) > 0
+    rng = np.random.default_rng(3)
+    for _ in range(300):
+        L, nv = int(rng.integers(1, 64)), int(rng.integers(0, 5000))
+        r = float(rng.random())
+        d = _desc(L=L, N=nv + 5, N_v=nv)
+        assert lib.tgvkv_vision_budget_total(ref(d), r) == oracle.vision_budget_total(r, nv, L)

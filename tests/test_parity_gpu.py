@@ -1,0 +1,249 @@
+"""GPU parity: the CUDA path through the C ABI against the fp64 oracle.
+
+Small cases (several row and key tiles, ragged tails, grouped-query heads,
+interleaved text, d = 64 and 128, edge cases) are checked in full; the four
+model-shaped workloads at their full sizes are checked on sampled layers, with
+the launch configuration the benchmark times.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2606_03075_gb300 import synth
+
+import _parity as P
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def api():
+    assert torch.cuda.is_available(), "the GPU tests need a CUDA device"
+    from paper_2606_03075_gb300 import build
+    build.build()
+    from paper_2606_03075_gb300 import api as _api
+    return _api
+
+
+def _seg_video(frames, stamp, per_frame, head, tail):
+    s = [("text", head)]
+    for _ in range(frames):
+        s += [("text", stamp), ("vision", per_frame)]
+    return s + [("text", tail)]
+
+
+SMALL = {
+    "ragged_mha": synth.custom("ragged_mha", 3, 4, 4, 128,
+                               [("text", 13), ("vision", 150), ("text", 7), ("vision", 61),
+                                ("text", 40)], ratios=(0.05, 0.3)),
+    "ragged_gqa": synth.custom("ragged_gqa", 2, 12, 2, 128,
+                               [("text", 5), ("vision", 100), ("text", 9), ("vision", 77),
+                                ("text", 30)], window="all_text", weights="dirichlet",
+                               ratios=(0.1,)),
+    "d64_gqa": synth.custom("d64_gqa", 2, 8, 4, 64,
+                            [("text", 20), ("vision", 180), ("text", 70)], ratios=(0.2,)),
+    "video_small": synth.custom("video_small", 2, 4, 1, 128, _seg_video(8, 4, 40, 8, 16),
+                                window="all_text", weights="dirichlet", ratios=(0.05,)),
+    "wide_group": synth.custom("wide_group", 1, 32, 1, 128,
+                               [("text", 3), ("vision", 90), ("text", 9)], ratios=(0.5,)),
+}
+
+
+def _full_check(api, wl, ratio, inp=None):
+    inp = inp if inp is not None else synth.generate(wl, seed=0)
+    g = P.run_evict(api, wl, inp, ratio)
+    assert g["status"] == 0
+    ref = oracle.evict(inp["q"], inp["k"], inp["v"], inp["modality"], inp["text_pos"],
+                       inp["w"], ratio, wl.H_kv)
+    P.assert_close(g["scores"], ref["scores"], "scores")
+    P.assert_close(g["stat"], ref["stat"], "tvb_stat")
+    # budgets: exact from the GPU statistic; end to end they agree unless a
+    # quota sits within the statistic's tolerance of a rounding boundary
+    total = oracle.vision_budget_total(ratio, wl.N_v, wl.L)
+    assert g["budgets"].tolist() == oracle.tvb_budgets(g["stat"], total, wl.N_v)
+    assert int(g["budgets"].sum()) == total
+    if not np.array_equal(g["budgets"], ref["budgets"]):
+        q = total * ref["stat"] / ref["stat"].sum()
+        assert np.min(np.abs(q - np.round(q))) < 1e-2, (g["budgets"], ref["budgets"])
+    P.check_selection_and_compaction(wl, inp, g, list(range(wl.L)),
+                                     ref_scores=ref["scores"] if np.array_equal(
+                                         g["budgets"], ref["budgets"]) else None)
+    assert g["offsets"][-1] == wl.H_kv * (wl.L * wl.N_t + total)
+    return g, ref
+
+
+def test_tiny(api):
+    _full_check(api, synth.WORKLOADS["tiny"], 0.25)
+
+
+@pytest.mark.parametrize("name", sorted(SMALL))
+def test_small_layouts(api, name):
+    wl = SMALL[name]
+    for r in wl.ratios:
+        _full_check(api, wl, r)
+
+
+@pytest.mark.parametrize("ratio", [0.0, 1.0])
+def test_budget_extremes(api, ratio):
+    g, _ = _full_check(api, SMALL["ragged_mha"], ratio)
+    assert set(g["budgets"].tolist()) == ({0} if ratio == 0.0 else {SMALL["ragged_mha"].N_v})
+
+
+def test_no_vision_tokens(api):
+    wl = synth.custom("no_vision", 2, 2, 2, 64, [("text", 50)], ratios=(0.5,))
+    g, _ = _full_check(api, wl, 0.5)
+    assert g["scores"].size == 0 and np.all(g["stat"] == 0)
+
+
+def test_single_query_row(api):
+    wl = synth.custom("one_row", 2, 4, 2, 128,
+                      [("text", 7), ("vision", 130), ("text", 1)], ratios=(0.3,))
+    assert wl.n_win == 1
+    _full_check(api, wl, 0.3)
+
+
+def test_queries_before_any_vision(api):
+    """Query rows that precede every vision key: zero TV mass everywhere, so
+    the budgets split uniformly and the kept vision keys are the lowest
+    positions (all scores tie at zero)."""
+    wl = synth.custom("early", 3, 4, 4, 64, [("text", 30), ("vision", 64), ("text", 10)],
+                      window=10, ratios=(0.25,))
+    inp = synth.generate(wl, seed=1)
+    inp["text_pos"] = np.arange(10, dtype=np.int32) * 3
+    g, ref = _full_check(api, wl, 0.25, inp=inp)
+    assert np.all(g["stat"] == 0) and np.all(g["scores"] == 0)
+    assert g["budgets"].tolist() == oracle.tvb_budgets([0, 0, 0], 48, 64)
+
+
+def test_separate_calls_match_fused(api):
+    wl = SMALL["ragged_gqa"]
+    ratio = 0.1
+    inp = synth.generate(wl, seed=3)
+    dev = P.device_inputs(inp)
+    fused = P.run_evict(api, wl, inp, ratio, dev=dev)
+    desc = api.desc_for_workload(wl)
+    ws = api.new_workspace(desc)
+    out = api.alloc_outputs(desc, ratio)
+    api.tgvkv_score(desc, dev["q"], dev["k"], dev["modality"], dev["text_pos"], dev["w"],
+                    out.scores, out.tvb_stat, ws)
+    api.tgvkv_budget(desc, out.tvb_stat, ratio, out.budgets, ws)
+    api.tgvkv_select(desc, out.scores, out.budgets, dev["modality"], out.offsets, out.idx, ws)
+    api.tgvkv_compact(desc, dev["k"], dev["v"], out.offsets, out.idx, out.k_out, out.v_out, ws)
+    assert api.tgvkv_status(ws) == 0
+    rows = api.tgvkv_retained_rows(desc, ratio)
+    np.testing.assert_array_equal(out.scores.cpu().numpy(), fused["scores"])
+    np.testing.assert_array_equal(out.tvb_stat.cpu().numpy(), fused["stat"])
+    np.testing.assert_array_equal(out.idx[:rows].cpu().numpy(), fused["idx"])
+    np.testing.assert_array_equal(out.k_out[:rows].view(torch.int16).cpu().numpy(), fused["k_out"])
+
+
+def test_repeat_calls_are_deterministic(api):
+    wl = SMALL["video_small"]
+    inp = synth.generate(wl, seed=4)
+    dev = P.device_inputs(inp)
+    a = P.run_evict(api, wl, inp, 0.05, dev=dev)
+    b = P.run_evict(api, wl, inp, 0.05, dev=dev)
+    for key in ("scores", "stat", "budgets", "offsets", "idx", "k_out", "v_out"):
+        np.testing.assert_array_equal(a[key], b[key], err_msg=key)
+
+
+# ---------------------------------------------------------------- single steps
+def test_budget_kernel_exact(api):
+    """TVB budgets from crafted statistics, including exact ties, zeros and caps."""
+    cases = [([0.5, 0.3, 0.2], 7, 100), ([1.0, 1.0, 1.0], 4, 100), ([0.9, 0.05, 0.05], 6, 3),
+             ([0.0, 0.0, 0.0, 0.0], 6, 10), ([0.0, 2.0, 1.0], 6, 10), ([3.0, 1.0], 8, 4)]
+    rng = np.random.default_rng(0)
+    for _ in range(40):
+        L = int(rng.integers(1, 40))
+        cap = int(rng.integers(1, 300))
+        stat = (rng.random(L) ** 2).astype(np.float32)
+        stat[rng.random(L) < 0.2] = 0.0
+        cases.append((stat.tolist(), int(rng.integers(0, L * cap + 1)), cap))
+    for stat, total, cap in cases:
+        L = len(stat)
+        ratio = total / float(cap * L)
+        # pick a ratio whose rounded total is `total`
+        desc = api.make_desc(L, 1, 1, 64, cap, cap, 1)
+        if api.tgvkv_vision_budget_total(desc, ratio) != total:
+            ratio = (total + 0.25) / float(cap * L)
+        assert api.tgvkv_vision_budget_total(desc, ratio) == total
+        s = torch.tensor(np.asarray(stat, np.float32), device="cuda")
+        b = torch.empty(L, dtype=torch.int32, device="cuda")
+        ws = api.new_workspace(desc)
+        api.tgvkv_budget(desc, s, ratio, b, ws)
+        assert api.tgvkv_status(ws) == 0
+        want = oracle.tvb_budgets(np.asarray(stat, np.float32).astype(np.float64), total, cap)
+        assert b.cpu().tolist() == want, (stat, total, cap)
+
+
+def test_select_kernel_ties_exact(api):
+    rng = np.random.default_rng(5)
+    for n, L, H in [(300, 3, 2), (2000, 2, 3), (5000, 1, 1)]:
+        modality = (rng.random(n) < 0.8).astype(np.uint8)
+        nv = int(modality.sum())
+        scores = (np.round(rng.random((L, H, nv)) * 16) / 16).astype(np.float32)
+        budgets = rng.integers(0, nv + 1, L).astype(np.int32)
+        budgets[0] = nv
+        if L > 1:
+            budgets[1] = 0
+        desc = api.make_desc(L, H, H, 64, n, nv, 1)
+        ws = api.new_workspace(desc)
+        off = torch.empty(L * H + 1, dtype=torch.int64, device="cuda")
+        idx = torch.empty(L * H * n, dtype=torch.int32, device="cuda")
+        api.tgvkv_select(desc, torch.from_numpy(scores).cuda(), torch.from_numpy(budgets).cuda(),
+                         torch.from_numpy(modality).cuda(), off, idx, ws)
+        assert api.tgvkv_status(ws) == 0
+        o_off, o_idx = oracle.tpr_select(scores, budgets, modality)
+        np.testing.assert_array_equal(off.cpu().numpy(), o_off)
+        np.testing.assert_array_equal(idx[:o_off[-1]].cpu().numpy(), o_idx)
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_compact_kernel_bit_exact(api, d):
+    rng = np.random.default_rng(d)
+    L, H, n = 3, 5, 77
+    k = rng.integers(-2 ** 15, 2 ** 15, (L, H, n, d)).astype(np.int16)
+    v = rng.integers(-2 ** 15, 2 ** 15, (L, H, n, d)).astype(np.int16)
+    sets = []
+    for lg in range(L * H):
+        m = int(rng.integers(0, n + 1)) if lg % 4 else (0 if lg % 8 == 0 else n)
+        sets.append(np.sort(rng.choice(n, m, replace=False)))
+    off = np.cumsum([0] + [s.size for s in sets]).astype(np.int64)
+    idx = np.concatenate(sets).astype(np.int32)
+    desc = api.make_desc(L, H, H, d, n, 0, 1)
+    ws = api.new_workspace(desc)
+    rows = max(int(off[-1]), 1)
+    ko = torch.zeros((rows, d), dtype=torch.int16, device="cuda")
+    vo = torch.zeros((rows, d), dtype=torch.int16, device="cuda")
+    api.tgvkv_compact(desc, torch.from_numpy(k).cuda(), torch.from_numpy(v).cuda(),
+                      torch.from_numpy(off).cuda(), torch.from_numpy(idx).cuda(), ko, vo, ws)
+    assert api.tgvkv_status(ws) == 0
+    rk, rv = oracle.compact(k, v, off, idx.astype(np.int64))
+    np.testing.assert_array_equal(ko[:off[-1]].cpu().numpy(), rk)
+    np.testing.assert_array_equal(vo[:off[-1]].cpu().numpy(), rv)
+
+
+# ---------------------------------------------------------------- full sizes
+FULL = [("llava15", 0.05, (0, 31)), ("llava15", 0.20, (17,)), ("next", 0.05, (0, 31)),
+        ("qwen25", 0.05, (13,)), ("video", 0.05, (27,))]
+
+
+@pytest.mark.parametrize("name,ratio,layers", FULL)
+def test_full_size_sampled(api, name, ratio, layers):
+    wl = synth.WORKLOADS[name]
+    inp = synth.generate(wl, seed=0)
+    g = P.run_evict(api, wl, inp, ratio)
+    assert g["status"] == 0
+    layers = list(layers)
+    ref_s, ref_t = P.oracle_scores(wl, inp, layers)
+    P.assert_close(g["scores"][layers], ref_s, f"{name} scores")
+    P.assert_close(g["stat"][layers], ref_t, f"{name} tvb_stat")
+    total = oracle.vision_budget_total(ratio, wl.N_v, wl.L)
+    assert g["budgets"].tolist() == oracle.tvb_budgets(g["stat"], total, wl.N_v)
+    assert np.all(g["stat"] > 0)
+    P.check_selection_and_compaction(wl, inp, g, layers, ref_scores=ref_s)
+    assert g["offsets"][-1] == wl.H_kv * (wl.L * wl.N_t + total)
+    assert np.all(np.diff(g["offsets"]) == np.repeat(wl.N_t + g["budgets"], wl.H_kv))
