@@ -1,0 +1,471 @@
+#!/usr/bin/env python
+"""Benchmark of the TGV-KV eviction step (score + budget + select + compact).
+
+Prints ONE JSON line on stdout (rank 0).  Metric: eviction microseconds per
+decoder layer for the fused tgvkv_evict over all layers of one request, plus
+the achieved HBM bandwidth of the step and the roofline of its dominant kernel.
+
+  python bench.py [--gpus N --steps K --warmup W] [--config llava15 --ratio 0.05]
+  python bench.py --impl reference ...   (the fp64 CPU oracle, same metric)
+
+Multi-GPU (torchrun, one rank per GPU): every rank runs its own replica of the
+workload (the step has no data-path exchange); the timed region is bracketed by
+a barrier and synchronisation and the max over ranks is reported.
+"""
+import argparse
+import ctypes
+import hashlib
+import json
+import math
+import os
+import statistics
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2606_03075_gb300 import synth  # noqa: E402
+
+METRIC = "eviction µs/layer and achieved HBM GB/s vs peak (score+budget+select+compact)"
+UNIT = "µs/layer"
+L2_BYTES = 129 * 2 ** 20
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="tgvkv", choices=["tgvkv", "reference"])
+    ap.add_argument("--config", default="llava15", choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--ratio", type=float, default=None)
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="wall-clock target of the oracle CPU-baseline sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+# --------------------------------------------------------------------------
+# workload description and algorithmic byte counts
+# --------------------------------------------------------------------------
+def workload_config(wl, ratio):
+    return {"workload": f"{wl.name}: L={wl.L} H_q/H_kv={wl.H_q}/{wl.H_kv} d={wl.d} "
+                        f"N={wl.N} (N_v={wl.N_v}, N_t={wl.N_t}) query rows={wl.n_win} "
+                        f"budget r={ratio} of vision KV",
+            "L": wl.L, "H_q": wl.H_q, "H_kv": wl.H_kv, "head_dim": wl.d, "N": wl.N,
+            "N_v": wl.N_v, "n_win": wl.n_win, "ratio": ratio, "weights": wl.weights,
+            "keys": wl.keys}
+
+
+def budget_total(wl, ratio):
+    return int(math.floor(ratio * float(wl.N_v * wl.L) + 0.5))
+
+
+def step_bytes(wl, ratio):
+    """Roofline bytes of one step: K read once + compacted K/V written."""
+    rows = wl.H_kv * (wl.L * wl.N_t + budget_total(wl, ratio))
+    k_read = wl.L * wl.H_kv * wl.N * wl.d * 2
+    kv_written = 2 * rows * wl.d * 2
+    return k_read + kv_written, rows
+
+
+def stage_bytes(wl, ratio):
+    """Algorithmic bytes of each kernel launch (all layers)."""
+    _, rows = step_bytes(wl, ratio)
+    k = wl.L * wl.H_kv * wl.N * wl.d * 2
+    q = wl.L * wl.H_q * wl.n_win * wl.d * 2
+    scores = wl.L * wl.H_kv * wl.N_v * 4
+    return {
+        "score": k + q + scores,
+        "budget": 8 * wl.L,
+        "select": scores + 4 * rows + 8 * (wl.L * wl.H_kv + 1),
+        "compact": 4 * rows * wl.d * 2 + 4 * rows,
+    }
+
+
+KERNEL_SOURCES = {"score": "score_stream.cu", "budget": "budget.cu", "select": "select.cu",
+                  "compact": "compact.cu"}
+
+
+def source_hash(stage):
+    path = os.path.join(ROOT, "paper_2606_03075_gb300", "csrc", KERNEL_SOURCES[stage])
+    with open(path, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def recorded_traffic(stage, workload):
+    """DRAM bytes per launch from a committed ncu capture, if the kernel source
+    is unchanged since the capture."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        rec = json.load(open(path))[stage][workload]
+    except (OSError, KeyError, ValueError):
+        return None
+    return rec["dram_bytes_per_launch"] if rec.get("source_sha") == source_hash(stage) else None
+
+
+def measured_peaks():
+    try:
+        return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))), "measured"
+    except (OSError, ValueError):
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}, "fallback"
+
+
+# --------------------------------------------------------------------------
+# clocks during the timed region (NVML through ctypes; nvidia-smi fallback)
+# --------------------------------------------------------------------------
+_REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+            0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
+
+
+class ClockSampler:
+    def __init__(self, torch_dev):
+        self.samples, self.reasons, self.max_mhz, self.ok = [], set(), None, False
+        self._stop = threading.Event()
+        try:
+            self.nvml = ctypes.CDLL("libnvidia-ml.so.1")
+            if self.nvml.nvmlInit_v2() != 0:
+                return
+            self.h = ctypes.c_void_p()
+            got = False
+            try:
+                import torch
+                pr = torch.cuda.get_device_properties(torch_dev)
+                bus = f"{pr.pci_domain_id:08x}:{pr.pci_bus_id:02x}:{pr.pci_device_id:02x}.0"
+                got = self.nvml.nvmlDeviceGetHandleByPciBusId_v2(bus.encode(), ctypes.byref(self.h)) == 0
+            except Exception:
+                got = False
+            if not got:
+                vis = os.environ.get("CUDA_VISIBLE_DEVICES", "0").split(",")[0]
+                idx = int(vis) if vis.isdigit() else 0
+                if self.nvml.nvmlDeviceGetHandleByIndex_v2(idx, ctypes.byref(self.h)) != 0:
+                    return
+            m = ctypes.c_uint()
+            if self.nvml.nvmlDeviceGetMaxClockInfo(self.h, 1, ctypes.byref(m)) == 0:
+                self.max_mhz = m.value
+            self.ok = True
+        except OSError:
+            self.ok = False
+
+    def _run(self):
+        c, r = ctypes.c_uint(), ctypes.c_ulonglong()
+        get_r = getattr(self.nvml, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            self.nvml.nvmlDeviceGetCurrentClocksThrottleReasons
+        while not self._stop.is_set():
+            if self.nvml.nvmlDeviceGetClockInfo(self.h, 1, ctypes.byref(c)) == 0:
+                self.samples.append(c.value)
+            if get_r(self.h, ctypes.byref(r)) == 0:
+                for bit, name in _REASONS.items():
+                    if r.value & bit:
+                        self.reasons.add(name)
+            time.sleep(0.002)
+
+    def __enter__(self):
+        if self.ok:
+            self.t = threading.Thread(target=self._run, daemon=True)
+            self.t.start()
+        return self
+
+    def __exit__(self, *a):
+        if self.ok:
+            self._stop.set()
+            self.t.join()
+
+    def summary(self):
+        if not self.ok or not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": self.max_mhz, "reasons": sorted(self.reasons),
+                    "samples": len(self.samples), "source": "nvml unavailable"}
+        return {"sm_mhz": statistics.median(self.samples), "sm_max_mhz": self.max_mhz,
+                "reasons": sorted(self.reasons), "samples": len(self.samples), "source": "nvml"}
+
+
+# --------------------------------------------------------------------------
+# CPU baseline: the oracle on a bounded sample of the workload
+# --------------------------------------------------------------------------
+def oracle_unit(wl, layer_inputs, l, g, ratio):
+    """The oracle's work for one (layer, KV head): Eq. 2/6/8 scores of its G
+    query heads, a TVB split, TPR selection and the compaction gather."""
+    import numpy as np
+    import oracle
+    q, k, v, w = layer_inputs
+    G = wl.G
+    scale = 1.0 / math.sqrt(wl.d)
+    qq = oracle.widen_bf16(q[g * G:(g + 1) * G])[None]
+    kk = oracle.widen_bf16(k[g:g + 1])[None]
+    s, st = oracle.twr_scores_tvb_stat(qq, kk, wl.modality, wl.text_pos, w[None].astype(np.float64),
+                                       scale, 1)
+    total = budget_total(wl, ratio)
+    budgets = oracle.tvb_budgets(np.full(wl.L, st[0]), total, wl.N_v)
+    off, idx = oracle.tpr_select(s, budgets[l:l + 1], wl.modality)
+    oracle.compact(k[None, g:g + 1], v[None, g:g + 1], off, idx)
+
+
+def run_cpu_baseline(wl, ratio, seed, seconds):
+    units, spent = 0, 0.0
+    for l in range(wl.L):
+        layer = synth.draw_layer(wl, seed, l)
+        for g in range(wl.H_kv):
+            t = time.perf_counter()
+            oracle_unit(wl, layer, l, g, ratio)
+            spent += time.perf_counter() - t
+            units += 1
+            if spent > seconds:
+                break
+        if spent > seconds:
+            break
+    us_per_layer = spent / units * wl.H_kv * 1e6
+    return {"value": us_per_layer, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"{units} (layer, KV head) units of {wl.name} in {spent:.1f} s "
+                      f"(fp64 numpy; BLAS may use all {os.cpu_count()} cores), scaled by "
+                      f"H_kv={wl.H_kv} per layer"}
+
+
+# --------------------------------------------------------------------------
+# reference arm: the oracle, timed per step on a bounded sample
+# --------------------------------------------------------------------------
+def run_reference(args, rank, world):
+    if rank != 0:
+        return 0
+    wl = synth.WORKLOADS[args.config]
+    ratio = args.ratio if args.ratio is not None else wl.ratios[0]
+    units = [(l, g) for l in range(wl.L) for g in range(wl.H_kv)]
+    cache = {}
+
+    def step(s):
+        l, g = units[s % len(units)]
+        if l not in cache:
+            cache.clear()
+            cache[l] = synth.draw_layer(wl, args.seed, l)
+        t = time.perf_counter()
+        oracle_unit(wl, cache[l], l, g, ratio)
+        return time.perf_counter() - t
+
+    for s in range(args.warmup):
+        step(s)
+    times = [step(args.warmup + s) for s in range(args.steps)]
+    mean = sum(times) / len(times)
+    value = mean * wl.H_kv * 1e6
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": mean * 1e3, "higher_is_better": False, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": workload_config(wl, ratio),
+            "cpu_baseline": {"kind": "oracle", "cores": os.cpu_count(), "value": value,
+                             "unit": UNIT,
+                             "sample": f"each step = one (layer, KV head) unit of {wl.name} "
+                                       f"(scores of its {wl.G} query heads, TVB split, TPR "
+                                       f"select, gather), fp64 numpy; µs/layer = step "
+                                       f"time x H_kv={wl.H_kv}"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# --------------------------------------------------------------------------
+# GPU arm
+# --------------------------------------------------------------------------
+def main():
+    args = parse()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if args.impl == "reference":
+        return run_reference(args, rank, world)
+
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    from paper_2606_03075_gb300 import build
+    build.build()
+    from paper_2606_03075_gb300 import api
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+
+    wl = synth.WORKLOADS[args.config]
+    ratio = args.ratio if args.ratio is not None else wl.ratios[0]
+    desc = api.desc_for_workload(wl)
+    inp = synth.generate(wl, seed=args.seed + rank)
+    in_bytes = sum(wl.input_bytes().values())
+    n_sets = max(2, math.ceil(2 * L2_BYTES / in_bytes) + 1)
+
+    def upload(a, dtype=None):
+        t = torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+        return t.view(dtype) if dtype is not None else t
+
+    sets = []
+    for i in range(n_sets):
+        sets.append(dict(q=upload(inp["q"], torch.bfloat16), k=upload(inp["k"], torch.bfloat16),
+                         v=upload(inp["v"], torch.bfloat16), modality=upload(inp["modality"]),
+                         text_pos=upload(inp["text_pos"]), w=upload(inp["w"])))
+    ws = api.new_workspace(desc, dev)
+    out = api.alloc_outputs(desc, ratio, dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def evict(s):
+        x = sets[s % n_sets]
+        api.tgvkv_evict(desc, x["q"], x["k"], x["v"], x["modality"], x["text_pos"], x["w"],
+                        ratio, out, ws, stream)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    # ---- warm-up, then the timed region (fused path)
+    for s in range(args.warmup):
+        evict(s)
+    if api.tgvkv_status(ws, stream) != 0:
+        raise RuntimeError("device status bits set during warm-up")
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    barrier()
+    with ClockSampler(dev) as clocks:
+        t_wall = time.perf_counter()
+        for s in range(args.steps):
+            ev[s][0].record(stream)
+            evict(args.warmup + s)
+            ev[s][1].record(stream)
+        barrier()
+        t_wall = time.perf_counter() - t_wall
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    region_ms = ev[0][0].elapsed_time(ev[-1][1])
+    if api.tgvkv_status(ws, stream) != 0:
+        raise RuntimeError("device status bits set in the timed region")
+    region = torch.tensor([region_ms], device=dev, dtype=torch.float64)
+    if world > 1:
+        dist.all_reduce(region, op=dist.ReduceOp.MAX)
+    region_ms = float(region.item())
+    us_per_layer = region_ms * 1e3 / (args.steps * wl.L * world)
+
+    # ---- per-stage breakdown (the four entry points with events between them)
+    stages = ["score", "budget", "select", "compact"]
+    sev = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
+    barrier()
+    for s in range(args.steps):
+        x = sets[s % n_sets]
+        e = sev[s]
+        e[0].record(stream)
+        api.tgvkv_score(desc, x["q"], x["k"], x["modality"], x["text_pos"], x["w"], out.scores,
+                        out.tvb_stat, ws, stream)
+        e[1].record(stream)
+        api.tgvkv_budget(desc, out.tvb_stat, ratio, out.budgets, ws, stream)
+        e[2].record(stream)
+        api.tgvkv_select(desc, out.scores, out.budgets, x["modality"], out.offsets, out.idx, ws,
+                         stream)
+        e[3].record(stream)
+        api.tgvkv_compact(desc, x["k"], x["v"], out.offsets, out.idx, out.k_out, out.v_out, ws,
+                          stream)
+        e[4].record(stream)
+    barrier()
+    stage_ms = {st: statistics.mean(sev[s][i].elapsed_time(sev[s][i + 1]) for s in range(args.steps))
+                for i, st in enumerate(stages)}
+
+    # ---- end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        pin = {k: torch.from_numpy(np.ascontiguousarray(inp[k])).pin_memory()
+               for k in ("q", "k", "v", "modality", "text_pos", "w")}
+        rows = api.tgvkv_retained_rows(desc, ratio)
+        host_out = dict(k_out=torch.empty((rows, wl.d), dtype=torch.bfloat16).pin_memory(),
+                        v_out=torch.empty((rows, wl.d), dtype=torch.bfloat16).pin_memory(),
+                        idx=torch.empty(rows, dtype=torch.int32).pin_memory(),
+                        offsets=torch.empty(wl.L * wl.H_kv + 1, dtype=torch.int64).pin_memory(),
+                        budgets=torch.empty(wl.L, dtype=torch.int32).pin_memory())
+        x = sets[0]
+        dst = dict(q=x["q"].view(torch.int16), k=x["k"].view(torch.int16),
+                   v=x["v"].view(torch.int16), modality=x["modality"], text_pos=x["text_pos"],
+                   w=x["w"])
+        h2d = sum(pin[k].numel() * pin[k].element_size() for k in pin)
+        d2h = sum(t.numel() * t.element_size() for t in host_out.values())
+        n_e2e = max(3, min(args.steps, 200))
+
+        def e2e_step():
+            for key in pin:
+                dst[key].copy_(pin[key], non_blocking=True)
+            api.tgvkv_evict(desc, x["q"], x["k"], x["v"], x["modality"], x["text_pos"], x["w"],
+                            ratio, out, ws, stream)
+            host_out["k_out"].copy_(out.k_out[:rows], non_blocking=True)
+            host_out["v_out"].copy_(out.v_out[:rows], non_blocking=True)
+            host_out["idx"].copy_(out.idx[:rows], non_blocking=True)
+            host_out["offsets"].copy_(out.offsets, non_blocking=True)
+            host_out["budgets"].copy_(out.budgets, non_blocking=True)
+
+        for _ in range(3):
+            e2e_step()
+        barrier()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(n_e2e):
+            e2e_step()
+        b.record(stream)
+        barrier()
+        e2e_ms = torch.tensor([a.elapsed_time(b)], device=dev, dtype=torch.float64)
+        if world > 1:
+            dist.all_reduce(e2e_ms, op=dist.ReduceOp.MAX)
+        e2e = {"value": float(e2e_ms.item()) * 1e3 / (n_e2e * wl.L * world), "unit": UNIT,
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n_e2e,
+               "path": "pinned host -> tgvkv_evict (C ABI) -> pinned host, one stream"}
+
+    # ---- roofline of the dominant kernel and of the whole step
+    peaks, peak_src = measured_peaks()
+    hbm_peak = float(peaks["hbm_gbs"])
+    sb = stage_bytes(wl, ratio)
+    dom = max(stages, key=lambda s: stage_ms[s])
+    achieved = sb[dom] / (stage_ms[dom] * 1e-3) / 1e9
+    traffic = recorded_traffic(dom, wl.name)
+    sbytes, rows = step_bytes(wl, ratio)
+    step_gbs = sbytes * args.steps * world / (region_ms * 1e-3) / 1e9
+
+    line = None
+    if rank == 0:
+        cpu = None
+        if world == 1 and not args.no_cpu_baseline:
+            cpu = run_cpu_baseline(wl, ratio, args.seed, args.cpu_seconds)
+        line = {
+            "metric": METRIC, "value": us_per_layer, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": region_ms / args.steps, "higher_is_better": False,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16->f32",
+            "data": "synthetic",
+            "config": dict(workload_config(wl, ratio),
+                           l2="inputs larger than L2: %d rotating input sets of %.0f MB "
+                              "(L2 %d MB)" % (n_sets, in_bytes / 1e6, L2_BYTES >> 20),
+                           parallelism=f"replicas x{world}"),
+            "hbm_step": {"bytes_per_step": sbytes, "bytes_per_layer": sbytes / wl.L,
+                         "gbs": step_gbs, "peak": hbm_peak, "frac": step_gbs / hbm_peak,
+                         "definition": "K read once + compacted K/V written, per step"},
+            "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": hbm_peak,
+                         "unit": "GB/s", "frac": achieved / hbm_peak, "traffic": traffic,
+                         "bytes_per_launch": sb[dom], "launch_ms": stage_ms[dom],
+                         "peak_source": f"{peak_src} hbm_gbs (MEASURED_PEAKS.json)"},
+            "stage_ms": stage_ms,
+            "step_ms_median": statistics.median(step_ms),
+            "wall_s_timed_region": t_wall,
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "gpu_launches": 4 * args.steps,
+            "clocks": clocks.summary(),
+        }
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+    if line is not None:
+        print(json.dumps(line), flush=True)
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())
