@@ -161,6 +161,37 @@ int tgvkv_status(void* workspace, void* stream);
 /* Message of the last error returned on the calling thread ("" if none). */
 const char* tgvkv_last_error(void);
 
+/* tgvkv_score without a caller workspace (the paper has no counterpart; this
+ * is a deployment variant of tgvkv_score).
+ *
+ * For callers that are handed only input and output buffers and cannot
+ * allocate device memory themselves: for example a plugin inside an inference
+ * runtime that owns all device memory and passes its operators no workspace,
+ * or a latency-critical path where cudaMalloc's implicit synchronisation is
+ * not allowed.  The scratch this call needs (completion counters, per-tile
+ * partial scores and TV masses) lives in a fixed array of
+ * TGVKV_NOALLOC_SCRATCH_BYTES inside the library; every GPU that loads the
+ * library holds that array until the process exits.  Nothing is allocated.
+ *
+ * Same arguments and results as tgvkv_score, minus the workspace.
+ * - A problem whose scratch exceeds TGVKV_NOALLOC_SCRATCH_BYTES (see
+ *   tgvkv_workspace_size) is rejected with TGVKV_ERR_UNSUPPORTED before any
+ *   launch.
+ * - The first call on each device looks up the array's device address (with
+ *   that device current) and caches it; make that first call before any
+ *   stream capture.
+ * - All calls share the one array.  Each call clears the parts that must start
+ *   at zero; calls whose work overlaps on the GPU (different streams, or
+ *   different host threads, on one device) race on the array and must be
+ *   serialised by the caller.
+ * - The device status word is kept in the array and cleared by every call, so
+ *   data-dependent input faults are skipped (never out of bounds) but not
+ *   reported; use tgvkv_score with a workspace to read them. */
+#define TGVKV_NOALLOC_SCRATCH_BYTES (8u << 20)
+int tgvkv_score_noalloc(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* k,
+                        const uint8_t* modality, const int32_t* text_pos, const float* w,
+                        float* scores, float* tvb_stat, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -41,6 +41,8 @@ SIGNATURES = {
     "tgvkv_workspace_init": (c_int, [_P, c_void_p, c_void_p]),
     "tgvkv_status": (c_int, [c_void_p, c_void_p]),
     "tgvkv_last_error": (c_char_p, []),
+    "tgvkv_score_noalloc": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                    c_void_p, c_void_p, c_void_p]),
 }
 
 _lib = None

@@ -5,6 +5,8 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <mutex>
+
 #include "common.cuh"
 #include "launch.h"
 #include "tgvkv.h"
@@ -294,3 +296,66 @@ int tgvkv_status(void* workspace, void* stream) {
 const char* tgvkv_last_error(void) { return g_last_error; }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// tgvkv_score_noalloc: tgvkv_score with its scratch in a fixed device array,
+// for callers that receive only input/output buffers and may not allocate.
+// ---------------------------------------------------------------------------
+namespace {
+
+// The scratch of every tgvkv_score_noalloc call on a device.  It keeps the
+// previous call's contents; the call clears what must start at zero.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[TGVKV_NOALLOC_SCRATCH_BYTES];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mutex;
+void* g_noalloc_ptr[kMaxDevices] = {};
+
+// Device address of g_noalloc_scratch on the current device, looked up once per
+// device.  The name is a host-side stand-in: only this address may be given to
+// a kernel.
+int noalloc_scratch(void** out) {
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return tgvkv::cuda_fail(e, "cudaGetDevice");
+    if (dev < 0 || dev >= kMaxDevices)
+        return tgvkv::fail(TGVKV_ERR_UNSUPPORTED, "device ordinal %d above %d", dev, kMaxDevices);
+    std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+    if (!g_noalloc_ptr[dev]) {
+        void* ptr = nullptr;
+        e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
+        if (e != cudaSuccess || ptr == nullptr)
+            return tgvkv::cuda_fail(e, "cudaGetSymbolAddress(static scratch)");
+        g_noalloc_ptr[dev] = ptr;
+    }
+    *out = g_noalloc_ptr[dev];
+    return TGVKV_OK;
+}
+
+}  // namespace
+
+extern "C" int tgvkv_score_noalloc(const tgvkv_desc* desc, const uint16_t* q_text,
+                                   const uint16_t* k, const uint8_t* modality,
+                                   const int32_t* text_pos, const float* w, float* scores,
+                                   float* tvb_stat, void* stream) {
+    Problem p{};
+    int rc = make_problem(desc, &p);
+    if (rc) return rc;
+    const WsLayout lay = layout_of(p);
+    if (lay.total > (size_t)TGVKV_NOALLOC_SCRATCH_BYTES)
+        return fail(TGVKV_ERR_UNSUPPORTED,
+                    "problem needs %zu bytes of scratch; the static scratch holds %u "
+                    "(use tgvkv_score with a caller workspace)",
+                    lay.total, (unsigned)TGVKV_NOALLOC_SCRATCH_BYTES);
+    void* scratch = nullptr;
+    if ((rc = noalloc_scratch(&scratch))) return rc;
+    rc = check_score_args(p, q_text, k, modality, text_pos, w, scores, tvb_stat, scratch);
+    if (rc) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    // the status word starts at zero for every call (the ticket counters are
+    // cleared by the score launch itself)
+    cudaError_t e = cudaMemsetAsync(static_cast<char*>(scratch) + lay.status, 0, sizeof(uint32_t), st);
+    if (e != cudaSuccess) return cuda_fail(e, "static scratch status clear");
+    rc = do_score(p, q_text, k, modality, text_pos, w, scores, tvb_stat, scratch, st);
+    return rc ? rc : ok();
+}
