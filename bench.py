@@ -91,7 +91,7 @@ def stage_bytes(wl, ratio):
     }
 
 
-KERNEL_SOURCES = {"score": "score_stream.cu", "budget": "budget.cu", "select": "select.cu",
+KERNEL_SOURCES = {"score": "score_tc.cu", "budget": "budget.cu", "select": "select.cu",
                   "compact": "compact.cu"}
 
 

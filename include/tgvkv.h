@@ -64,6 +64,7 @@ extern "C" {
 #define TGVKV_STATUS_INDEX        0x08u /* an index outside [0, N) reached compact */
 #define TGVKV_STATUS_COUNT        0x10u /* a retained set did not hold N_t + b_l rows */
 #define TGVKV_STATUS_TIMEOUT      0x20u /* a bounded on-chip wait gave up */
+#define TGVKV_STATUS_WEIGHT       0x40u /* a text weight is negative or not finite */
 
 /* ---- problem description --------------------------------------------- */
 typedef struct tgvkv_desc {
@@ -104,7 +105,7 @@ int64_t tgvkv_retained_rows(const tgvkv_desc* desc, double ratio);
  * k:        bf16 [L][H_kv][N][d]          (the key cache)
  * modality: uint8 [N], 1 = vision token, 0 = text token (same for all layers)
  * text_pos: int32 [n_win], strictly ascending positions in [0, N)
- * w:        fp32 text weights w~, row l at w + l * w_layer_stride, n_win floats
+ * w:        fp32 text weights w~ >= 0, row l at w + l * w_layer_stride, n_win floats
  * scores:   fp32 [L][H_kv][N_v]  (output)
  * tvb_stat: fp32 [L]             (output)
  * Arithmetic: bf16 products, fp32 accumulation and fp32 softmax. */

@@ -9,7 +9,7 @@ from . import synth  # noqa: F401
 
 STATUS_BITS = {
     0x01: "TEXT_POS", 0x02: "VISION_COUNT", 0x04: "BUDGET", 0x08: "INDEX",
-    0x10: "COUNT", 0x20: "TIMEOUT",
+    0x10: "COUNT", 0x20: "TIMEOUT", 0x40: "WEIGHT",
 }
 
 

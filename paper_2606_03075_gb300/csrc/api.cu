@@ -73,6 +73,9 @@ int make_problem(const tgvkv_desc* d, Problem* p) {
     if (rows > (1LL << 24)) return fail(TGVKV_ERR_UNSUPPORTED, "G * n_win = %lld too large", rows);
     if ((long long)d->L * d->H_kv > 65535)
         return fail(TGVKV_ERR_UNSUPPORTED, "L * H_kv above 65535");
+    if ((long long)d->L * d->H_kv * d->N >= (1LL << 31) ||
+        (long long)d->L * d->H_q * d->n_win >= (1LL << 31))
+        return fail(TGVKV_ERR_UNSUPPORTED, "K or Q holds 2^31 rows or more");
     p->L = d->L;
     p->H_q = d->H_q;
     p->H_kv = d->H_kv;

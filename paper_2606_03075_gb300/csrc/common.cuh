@@ -27,7 +27,7 @@ struct WsLayout {
     size_t total;
 };
 
-constexpr int kMaxN = 65536;     // key positions per head handled by one CTA's tile map
+constexpr int kMaxN = 32768;     // key positions per head (the per-CTA tile maps)
 constexpr int kMaxNv = 49152;    // vision keys held in shared memory by select
 constexpr int kMaxL = 1024;      // layers handled by the budget kernel
 
@@ -39,6 +39,13 @@ __device__ __forceinline__ void raise_status(uint32_t* status, uint32_t bits) {
 __device__ __forceinline__ float fast_exp2(float x) {
     float y;
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// log2(x) with the MUFU.LG2 unit (PTX lg2.approx.ftz.f32; lg2(0) = -inf).
+__device__ __forceinline__ float fast_log2(float x) {
+    float y;
+    asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
     return y;
 }
 

@@ -15,6 +15,13 @@ cudaError_t launch_score(const Problem& p, const uint16_t* q, const uint16_t* k,
                          float* scores, float* tvb_stat, char* ws, const WsLayout& lay,
                          cudaStream_t stream);
 
+// tcgen05 / TMA score kernel (score_tc.cu); launch_score clears the counters,
+// handles the empty cases and calls it.
+cudaError_t launch_score_tc(const Problem& p, const uint16_t* q, const uint16_t* k,
+                            const uint8_t* modality, const int32_t* text_pos, const float* w,
+                            float* scores, float* tvb_stat, char* ws, const WsLayout& lay,
+                            cudaStream_t stream);
+
 cudaError_t launch_budget(const Problem& p, const float* tvb_stat, long long total,
                           int32_t* budgets, uint32_t* status, cudaStream_t stream);
 

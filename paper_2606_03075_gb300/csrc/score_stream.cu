@@ -438,6 +438,13 @@ cudaError_t launch_score(const Problem& p, const uint16_t* q, const uint16_t* k,
         }
         return cudaMemsetAsync(tvb_stat, 0, sizeof(float) * (size_t)p.L, stream);
     }
+    return launch_score_tc(p, q, k, modality, text_pos, w, scores, tvb_stat, ws, lay, stream);
+}
+
+cudaError_t launch_score_stream(const Problem& p, const uint16_t* q, const uint16_t* k,
+                                const uint8_t* modality, const int32_t* text_pos, const float* w,
+                                float* scores, float* tvb_stat, char* ws, const WsLayout& lay,
+                                cudaStream_t stream) {
     if (p.d == 64)
         return launch_stream<64>(p, q, k, modality, text_pos, w, scores, tvb_stat, ws, lay, stream);
     return launch_stream<128>(p, q, k, modality, text_pos, w, scores, tvb_stat, ws, lay, stream);
