@@ -151,7 +151,10 @@ int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
                 void* workspace, void* stream);
 
 /* Zero `workspace` (asynchronously on `stream`).  Needed once after the
- * workspace is allocated; the calls keep it consistent afterwards. */
+ * workspace is allocated: the calls leave their completion counters at zero
+ * for the next call.  Zero it again after a call whose tgvkv_status reported
+ * TGVKV_STATUS_TIMEOUT, and never share one workspace between calls that may
+ * overlap on the GPU. */
 int tgvkv_workspace_init(const tgvkv_desc* desc, void* workspace, void* stream);
 
 /* Synchronise `stream`, then read and clear the device status word kept in

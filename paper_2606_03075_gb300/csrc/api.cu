@@ -41,7 +41,7 @@ WsLayout layout_of(const Problem& p) {
     WsLayout w;
     size_t o = 0;
     w.status = o;      o += round_up(sizeof(uint32_t));
-    w.tickets = o;     o += round_up(sizeof(uint32_t) * (size_t)(p.L * p.H_kv + p.L));
+    w.tickets = o;     o += round_up(sizeof(uint32_t) * ticket_words(p));
     w.stat_part = o;   o += round_up(sizeof(float) * (size_t)p.L * p.H_kv * (p.T > 0 ? p.T : 1));
     w.stat_head = o;   o += round_up(sizeof(float) * (size_t)p.L * p.H_kv);
     w.score_part = o;
@@ -70,7 +70,7 @@ int make_problem(const tgvkv_desc* d, Problem* p) {
     if (!(d->softmax_scale == d->softmax_scale) || isinf(d->softmax_scale))
         return fail(TGVKV_ERR_INVALID_ARG, "softmax_scale is not finite");
     const long long rows = (long long)(d->H_q / d->H_kv) * d->n_win;
-    if (rows > (1LL << 24)) return fail(TGVKV_ERR_UNSUPPORTED, "G * n_win = %lld too large", rows);
+    if (rows > 32768) return fail(TGVKV_ERR_UNSUPPORTED, "G * n_win = %lld above 32768", rows);
     if ((long long)d->L * d->H_kv > 65535)
         return fail(TGVKV_ERR_UNSUPPORTED, "L * H_kv above 65535");
     if ((long long)d->L * d->H_kv * d->N >= (1LL << 31) ||
@@ -258,12 +258,10 @@ int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
     cudaError_t e = launch_score(p, q_text, k, modality, text_pos, w, scores, tvb_stat,
                                  static_cast<char*>(workspace), lay, st);
     if (e != cudaSuccess) return cuda_fail(e, "score launch");
-    e = launch_budget(p, tvb_stat, budget_total(p, ratio), budgets, status, st);
-    if (e != cudaSuccess) return cuda_fail(e, "budget launch");
-    e = launch_select(p, scores, budgets, modality, offsets, idx, status, st);
-    if (e != cudaSuccess) return cuda_fail(e, "select launch");
-    e = launch_compact(p, k, v, offsets, idx, k_out, v_out, retained_rows(p, ratio), status, st);
-    if (e != cudaSuccess) return cuda_fail(e, "compact launch");
+    e = launch_budget_select_compact(p, scores, tvb_stat, budget_total(p, ratio), budgets,
+                                     modality, offsets, idx, k, v, k_out, v_out,
+                                     retained_rows(p, ratio), status, st);
+    if (e != cudaSuccess) return cuda_fail(e, "budget/select/compact launch");
     return ok();
 }
 
@@ -355,10 +353,12 @@ extern "C" int tgvkv_score_noalloc(const tgvkv_desc* desc, const uint16_t* q_tex
     rc = check_score_args(p, q_text, k, modality, text_pos, w, scores, tvb_stat, scratch);
     if (rc) return rc;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    // the status word starts at zero for every call (the ticket counters are
-    // cleared by the score launch itself)
+    // the status word and the completion counters start at zero for every call
     cudaError_t e = cudaMemsetAsync(static_cast<char*>(scratch) + lay.status, 0, sizeof(uint32_t), st);
-    if (e != cudaSuccess) return cuda_fail(e, "static scratch status clear");
+    if (e == cudaSuccess)
+        e = cudaMemsetAsync(static_cast<char*>(scratch) + lay.tickets, 0,
+                            sizeof(uint32_t) * ticket_words(p), st);
+    if (e != cudaSuccess) return cuda_fail(e, "static scratch clear");
     rc = do_score(p, q_text, k, modality, text_pos, w, scores, tvb_stat, scratch, st);
     return rc ? rc : ok();
 }

@@ -20,12 +20,18 @@ struct Problem {
 // Workspace layout (byte offsets into the caller's buffer).
 struct WsLayout {
     size_t status;      // uint32 status word
-    size_t tickets;     // uint32 [L*H_kv + L]: completion counters
+    size_t tickets;     // uint32 [ticket_words]: completion counters (heads, layers), work counter
     size_t stat_part;   // float [L*H_kv*T]: TV mass of one row tile
     size_t stat_head;   // float [L*H_kv]: TV mass of one KV head
     size_t score_part;  // float [L*H_kv*T*N_v]: scores of one row tile (T > 1)
     size_t total;
 };
+
+// Counters at the start of the workspace: one per KV head, one per layer, then
+// the score kernel's work counter and its done counter.
+__host__ __device__ inline size_t ticket_words(const Problem& p) {
+    return (size_t)p.L * p.H_kv + p.L + 2;
+}
 
 constexpr int kMaxN = 32768;     // key positions per head (the per-CTA tile maps)
 constexpr int kMaxNv = 49152;    // vision keys held in shared memory by select
@@ -49,33 +55,26 @@ __device__ __forceinline__ float fast_log2(float x) {
     return y;
 }
 
+// Packed pairs of fp32 (Blackwell f32x2 FMA-pipe instructions).
+union F2 {
+    float2 f;
+    unsigned long long u;
+};
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
+    F2 x, y, z, r;
+    x.f = a; y.f = b; z.f = c;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r.u) : "l"(x.u), "l"(y.u), "l"(z.u));
+    return r.f;
+}
+__device__ __forceinline__ float2 add2(float2 a, float2 b) {
+    F2 x, y, r;
+    x.f = a; y.f = b;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r.u) : "l"(x.u), "l"(y.u));
+    return r.f;
+}
+
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-// ---- Ampere-style async copy and warp MMA (used by the streaming score kernel)
-__device__ __forceinline__ void cp_async_16(uint32_t saddr, const void* gptr) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(saddr), "l"(gptr));
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N)); }
-
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
-                                        uint32_t& r3) {
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
-                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-                 : "r"(addr));
-}
-
-// D += A * B, m16n8k16, bf16 inputs, fp32 accumulate.
-__device__ __forceinline__ void mma_bf16_16816(float (&c)[4], const uint32_t (&a)[4], uint32_t b0,
-                                               uint32_t b1) {
-    asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
-        "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};\n"
-        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
 // Order-preserving map of an fp32 value to uint32 (larger float -> larger key).

@@ -10,17 +10,12 @@
 
 namespace tgvkv {
 
+// TWR scores + TVB statistic (score_tc.cu).  The completion counters in the
+// workspace must be zero on entry; the kernel leaves them zero.
 cudaError_t launch_score(const Problem& p, const uint16_t* q, const uint16_t* k,
                          const uint8_t* modality, const int32_t* text_pos, const float* w,
                          float* scores, float* tvb_stat, char* ws, const WsLayout& lay,
                          cudaStream_t stream);
-
-// tcgen05 / TMA score kernel (score_tc.cu); launch_score clears the counters,
-// handles the empty cases and calls it.
-cudaError_t launch_score_tc(const Problem& p, const uint16_t* q, const uint16_t* k,
-                            const uint8_t* modality, const int32_t* text_pos, const float* w,
-                            float* scores, float* tvb_stat, char* ws, const WsLayout& lay,
-                            cudaStream_t stream);
 
 cudaError_t launch_budget(const Problem& p, const float* tvb_stat, long long total,
                           int32_t* budgets, uint32_t* status, cudaStream_t stream);
@@ -28,6 +23,18 @@ cudaError_t launch_budget(const Problem& p, const float* tvb_stat, long long tot
 cudaError_t launch_select(const Problem& p, const float* scores, const int32_t* budgets,
                           const uint8_t* modality, int64_t* offsets, int32_t* idx,
                           uint32_t* status, cudaStream_t stream);
+
+// budget + select + gather fused (tgvkv_evict): one CTA per (layer, KV head)
+// derives all layer budgets from the TVB statistic, selects its set and
+// gathers its rows; falls back to the three separate kernels when the keys and
+// retained rows of a head do not fit in shared memory.
+cudaError_t launch_budget_select_compact(const Problem& p, const float* scores,
+                                         const float* tvb_stat, long long budget_total,
+                                         int32_t* budgets, const uint8_t* modality,
+                                         int64_t* offsets, int32_t* idx, const uint16_t* k,
+                                         const uint16_t* v, uint16_t* k_out, uint16_t* v_out,
+                                         long long capacity_rows, uint32_t* status,
+                                         cudaStream_t stream);
 
 cudaError_t launch_compact(const Problem& p, const uint16_t* k, const uint16_t* v,
                            const int64_t* offsets, const int32_t* idx, uint16_t* k_out,

@@ -1,21 +1,25 @@
 // TPR retention (Eq. 10, case b_l > N_t, vision budget b_l): one CTA per
 // (layer, KV head) keeps every text position and the b_l vision positions of
-// highest score, ties to the lower position, and writes them in ascending
-// position order.
+// highest score, ties to the lower position, in ascending position order --
+// and, in the fused form used by tgvkv_evict, gathers the retained K and V
+// rows straight away.
 //
-// Selection: the scores are mapped to order-preserving 32-bit keys in shared
-// memory; an MSB-first radix select (four 8-bit digits) finds the key T of the
-// b_l-th largest score and how many keys equal to T are still needed (k_eq).
-// A vision key is kept iff key > T, or key == T and it is among the first k_eq
-// such keys in position order.  One ordered pass over the positions then
-// emits text and kept vision positions through block prefix sums.
+// Selection: the scores become order-preserving 32-bit keys in shared memory;
+// an MSB-first radix select (four 8-bit digits) finds the key T of the b_l-th
+// largest score and how many keys equal to T are still needed (k_eq).  A
+// vision key is kept iff key > T, or key == T and it is among the first k_eq
+// such keys in position order.  Each thread then owns a contiguous range of
+// positions; three block prefix sums (vision keys, keys equal to T, kept
+// positions) give every kept position its output slot.
+#include "budget.cuh"
 #include "common.cuh"
 #include "launch.h"
 
 namespace tgvkv {
 namespace {
 
-constexpr int kThreads = 1024;
+constexpr int kThreads = 256;
+constexpr size_t kFusedSmemLimit = 200 * 1024; // keys + retained rows held for the gather
 
 // Exclusive prefix sum of x over the block; *total gets the block sum.
 __device__ __forceinline__ int block_exclusive_scan(int x, int* buf, int* total) {
@@ -29,7 +33,7 @@ __device__ __forceinline__ int block_exclusive_scan(int x, int* buf, int* total)
     if (lane == 31) buf[warp] = incl;
     __syncthreads();
     if (warp == 0) {
-        const int v = (lane < (int)(blockDim.x >> 5)) ? buf[lane] : 0;
+        const int v = (lane < kThreads / 32) ? buf[lane] : 0;
         int iv = v;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
@@ -46,11 +50,24 @@ __device__ __forceinline__ int block_exclusive_scan(int x, int* buf, int* total)
     return res;
 }
 
+constexpr size_t kBudgetBytes = (sizeof(BudgetScratch) + 15) & ~size_t(15);
+
+// COMPACT: also gather the retained rows.  FUSED_BUDGET: derive the budgets
+// from the TVB statistic (every CTA runs the same deterministic split; CTA 0
+// writes them out) instead of reading them.
+template <bool COMPACT, bool FUSED_BUDGET, int VPR>
 __global__ void __launch_bounds__(kThreads)
-tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __restrict__ budgets,
+tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __restrict__ budgets_in,
+                  const float* __restrict__ tvb_stat, long long budget_total,
+                  int32_t* __restrict__ budgets_out,
                   const uint8_t* __restrict__ modality, int64_t* __restrict__ offsets,
-                  int32_t* __restrict__ idx, uint32_t* __restrict__ status) {
-    extern __shared__ uint32_t keys[];  // [N_v]
+                  int32_t* __restrict__ idx, const uint4* __restrict__ k,
+                  const uint4* __restrict__ v, uint4* __restrict__ k_out,
+                  uint4* __restrict__ v_out, uint32_t* __restrict__ status) {
+    extern __shared__ __align__(16) unsigned char dyn_raw[];
+    BudgetScratch& bs = *reinterpret_cast<BudgetScratch*>(dyn_raw);
+    uint32_t* keys = reinterpret_cast<uint32_t*>(dyn_raw + (FUSED_BUDGET ? kBudgetBytes : 0));  // [N_v]
+    int* rows = reinterpret_cast<int*>(keys + p.N_v);       // [N_t + b] (gather form)
     __shared__ int hist[256];
     __shared__ int scan_buf[33];
     __shared__ uint32_t s_prefix;
@@ -60,6 +77,12 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
     const int lg = blockIdx.x, l = lg / p.H_kv, g = lg % p.H_kv;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 
+    const int32_t* budgets = budgets_in;
+    if (FUSED_BUDGET) {
+        tvb_budget_block(tvb_stat, p.L, budget_total, p.N_v, blockIdx.x == 0 ? budgets_out : nullptr,
+                         status, bs);
+        budgets = bs.result;
+    }
     int b = budgets[l];
     if (b < 0 || b > p.N_v) {
         if (tid == 0) raise_status(status, TGVKV_STATUS_BUDGET);
@@ -79,7 +102,7 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
         if (lg == p.L * p.H_kv - 1) offsets[lg + 1] = off + len;
     }
     const float* sc = scores + (size_t)lg * p.N_v;
-    for (int v = tid; v < p.N_v; v += kThreads) keys[v] = float_order_key(sc[v]);
+    for (int i = tid; i < p.N_v; i += kThreads) keys[i] = float_order_key(__ldg(sc + i));
     __syncthreads();
 
     // ---- radix select of the b-th largest key
@@ -87,11 +110,11 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
     int kk = b;
     if (b > 0) {
         for (int shift = 24; shift >= 0; shift -= 8) {
-            if (tid < 256) hist[tid] = 0;
+            hist[tid] = 0;   // kThreads == 256 bins
             __syncthreads();
             const uint32_t hi_mask = (shift == 24) ? 0u : (0xFFFFFFFFu << (shift + 8));
-            for (int v = tid; v < p.N_v; v += kThreads) {
-                const uint32_t key = keys[v];
+            for (int i = tid; i < p.N_v; i += kThreads) {
+                const uint32_t key = keys[i];
                 if ((key & hi_mask) == (prefix & hi_mask)) atomicAdd(&hist[(key >> shift) & 255], 1);
             }
             __syncthreads();
@@ -133,29 +156,106 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
     const uint32_t thr = prefix;
     const int k_eq = none ? 0 : kk;
 
-    // ---- ordered emission: text positions and kept vision positions
-    const long long off = s_off;
-    int vis_run = 0, eq_run = 0, keep_run = 0;
-    for (int base = 0; base < p.N; base += kThreads) {
-        const int j = base + tid;
-        const int is_vis = (j < p.N && modality[j] != 0) ? 1 : 0;
-        int tot;
-        const int vr = vis_run + block_exclusive_scan(is_vis, scan_buf, &tot);
-        vis_run += tot;
-        int is_eq = 0, is_gt = 0;
-        if (is_vis && vr < p.N_v) {
-            const uint32_t key = keys[vr];
-            is_gt = key > thr;
-            is_eq = key == thr;
-        }
-        const int er = eq_run + block_exclusive_scan(is_eq, scan_buf, &tot);
-        eq_run += tot;
-        const int keep = (j < p.N) && (!is_vis || (!none && (is_gt || (is_eq && er < k_eq))));
-        const int kr = keep_run + block_exclusive_scan(keep, scan_buf, &tot);
-        keep_run += tot;
-        if (keep && kr < len) idx[off + kr] = j;
+    // ---- ordered emission over per-thread position ranges
+    const int per = (p.N + kThreads - 1) / kThreads;
+    const int j0 = min(p.N, tid * per), j1 = min(p.N, j0 + per);
+    int nv = 0;
+    for (int j = j0; j < j1; ++j) nv += modality[j] != 0;
+    int tot;
+    const int vbase = block_exclusive_scan(nv, scan_buf, &tot);
+    int neq = 0;
+    if (!none) {
+        int vr = vbase;
+        for (int j = j0; j < j1; ++j)
+            if (modality[j] != 0) {
+                neq += (vr < p.N_v && keys[vr] == thr);
+                ++vr;
+            }
     }
-    if (tid == 0 && keep_run != len) raise_status(status, TGVKV_STATUS_COUNT);
+    const int ebase = block_exclusive_scan(neq, scan_buf, &tot);
+    // kept(j): text, or a vision key above T, or one of the first k_eq equal to T
+    auto scan_kept = [&](auto&& emit) {
+        int vr = vbase, er = ebase;
+        for (int j = j0; j < j1; ++j) {
+            bool keep = true;
+            if (modality[j] != 0) {
+                keep = false;
+                if (vr < p.N_v && !none) {
+                    const uint32_t key = keys[vr];
+                    if (key > thr) {
+                        keep = true;
+                    } else if (key == thr) {
+                        keep = er < k_eq;
+                        ++er;
+                    }
+                }
+                ++vr;
+            }
+            if (keep) emit(j);
+        }
+    };
+    int nkeep = 0;
+    scan_kept([&](int) { ++nkeep; });
+    const int kbase = block_exclusive_scan(nkeep, scan_buf, &tot);
+    const long long off = s_off;
+    {
+        int r = kbase;
+        scan_kept([&](int j) {
+            if (r < len) {
+                idx[off + r] = j;
+                if (COMPACT) rows[r] = j;
+            }
+            ++r;
+        });
+    }
+    if (tid == 0 && tot != len) raise_status(status, TGVKV_STATUS_COUNT);
+    if (!COMPACT) return;
+
+    // ---- gather the retained K and V rows (fused form)
+    __syncthreads();
+    constexpr int RPI = 32 / VPR;     // rows per warp per step
+    constexpr int UNROLL = 4;
+    const int n = min(len, tot);
+    const int sub = lane / VPR, vec = lane % VPR;
+    const size_t head = (size_t)lg * p.N;
+    for (int r0 = warp * RPI * UNROLL; r0 < n; r0 += (kThreads / 32) * RPI * UNROLL) {
+        uint4 kr[UNROLL], vr[UNROLL];
+#pragma unroll
+        for (int u = 0; u < UNROLL; ++u) {
+            const int r = r0 + u * RPI + sub;
+            if (r < n) {
+                const size_t src = (head + rows[r]) * VPR + vec;
+                kr[u] = __ldg(k + src);
+                vr[u] = __ldg(v + src);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < UNROLL; ++u) {
+            const int r = r0 + u * RPI + sub;
+            if (r < n) {
+                const size_t dst = (size_t)(off + r) * VPR + vec;
+                k_out[dst] = kr[u];
+                v_out[dst] = vr[u];
+            }
+        }
+    }
+}
+
+template <bool COMPACT, bool FUSED_BUDGET, int VPR>
+cudaError_t launch_sel(const Problem& p, const float* scores, const int32_t* budgets_in,
+                       const float* tvb_stat, long long budget_total, int32_t* budgets_out,
+                       const uint8_t* modality, int64_t* offsets, int32_t* idx,
+                       const uint16_t* k, const uint16_t* v, uint16_t* k_out, uint16_t* v_out,
+                       uint32_t* status, size_t smem, cudaStream_t stream) {
+    auto kern = tpr_select_kernel<COMPACT, FUSED_BUDGET, VPR>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    kern<<<p.L * p.H_kv, kThreads, smem, stream>>>(
+        p, scores, budgets_in, tvb_stat, budget_total, budgets_out, modality, offsets, idx,
+        reinterpret_cast<const uint4*>(k),
+        reinterpret_cast<const uint4*>(v), reinterpret_cast<uint4*>(k_out),
+        reinterpret_cast<uint4*>(v_out), status);
+    return cudaGetLastError();
 }
 
 }  // namespace
@@ -163,13 +263,32 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
 cudaError_t launch_select(const Problem& p, const float* scores, const int32_t* budgets,
                           const uint8_t* modality, int64_t* offsets, int32_t* idx,
                           uint32_t* status, cudaStream_t stream) {
-    const size_t smem = sizeof(uint32_t) * (size_t)p.N_v;
-    cudaError_t e = cudaFuncSetAttribute(tpr_select_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    tpr_select_kernel<<<p.L * p.H_kv, kThreads, smem, stream>>>(p, scores, budgets, modality,
-                                                                offsets, idx, status);
-    return cudaGetLastError();
+    return launch_sel<false, false, 16>(p, scores, budgets, nullptr, -1, nullptr, modality, offsets,
+                                        idx, nullptr, nullptr, nullptr, nullptr, status,
+                                        sizeof(uint32_t) * (size_t)p.N_v, stream);
+}
+
+cudaError_t launch_budget_select_compact(const Problem& p, const float* scores,
+                                         const float* tvb_stat, long long budget_total,
+                                         int32_t* budgets, const uint8_t* modality,
+                                         int64_t* offsets, int32_t* idx, const uint16_t* k,
+                                         const uint16_t* v, uint16_t* k_out, uint16_t* v_out,
+                                         long long capacity_rows, uint32_t* status,
+                                         cudaStream_t stream) {
+    const size_t smem = kBudgetBytes + sizeof(uint32_t) * ((size_t)p.N_v + (size_t)p.N);
+    if (smem > kFusedSmemLimit) {
+        cudaError_t e = launch_budget(p, tvb_stat, budget_total, budgets, status, stream);
+        if (e == cudaSuccess)
+            e = launch_select(p, scores, budgets, modality, offsets, idx, status, stream);
+        if (e != cudaSuccess) return e;
+        return launch_compact(p, k, v, offsets, idx, k_out, v_out, capacity_rows, status, stream);
+    }
+    if (p.d == 64)
+        return launch_sel<true, true, 8>(p, scores, nullptr, tvb_stat, budget_total, budgets,
+                                         modality, offsets, idx, k, v, k_out, v_out, status, smem,
+                                         stream);
+    return launch_sel<true, true, 16>(p, scores, nullptr, tvb_stat, budget_total, budgets, modality,
+                                      offsets, idx, k, v, k_out, v_out, status, smem, stream);
 }
 
 }  // namespace tgvkv
