@@ -119,6 +119,23 @@ __device__ __forceinline__ Item item_info(const Problem& p, const PSmem<D>& s, i
     return it;
 }
 
+// One 128 x 128 x D product into the accumulator at d_tmem: D/16 MMAs whose
+// operand descriptors differ from the tile's base descriptors by constants
+// (K offset of 32 bytes inside a 128-byte swizzle atom, 16 KB per 64 dims).
+// Pass A: S = Q K^T (TRANS = false); pass B: S^T = K Q^T.
+template <int D, bool TRANS>
+__device__ __forceinline__ void mma_kq(uint32_t d_tmem, uint64_t qd, uint64_t kd) {
+#pragma unroll
+    for (int kk = 0; kk < D / 16; ++kk) {
+        const uint64_t o = (uint64_t)((kk >> 2) * (BM * 64 * 2 / 16) + (kk & 3) * 2);
+        const uint64_t a = TRANS ? kd + o : qd + o, b = TRANS ? qd + o : kd + o;
+        if (kk == 0)
+            tc::mma_bf16_c<0>(d_tmem, a, b, IDESC);
+        else
+            tc::mma_bf16_c<1>(d_tmem, a, b, IDESC);
+    }
+}
+
 __device__ __forceinline__ int next_vis_tile(const int* vis_before, int kt, int n_tiles) {
     while (kt < n_tiles && vis_before[kt + 1] == vis_before[kt]) ++kt;
     return kt;
@@ -416,6 +433,12 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
 
     // ------------------------------------------------------------ MMA issuer
     if (warp == 1 && lane == 0) {
+        // shared-memory descriptors, computed once: the start-address field
+        // (16-byte units, < 2^14 inside 256 KB) takes plain additions
+        const uint64_t kdesc0 = tc::sdesc_k_sw128(smem_u32(&s.k[0][0][0]));
+        const uint64_t qdesc0 = tc::sdesc_k_sw128(smem_u32(&s.q[0][0][0]));
+        constexpr uint32_t KSTAGE_DESC = (uint32_t)(sizeof(s.k[0]) >> 4);
+        constexpr uint32_t QBUF_DESC = (uint32_t)(sizeof(s.q[0]) >> 4);
         int it = 0, qn = 0;
         int acc[NGRP] = {0, 0};
         bool ok = true;
@@ -438,7 +461,9 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
                 }
             }
             if (!ok) break;
-            const uint32_t qa0 = smem_u32(&s.q[qb0][0][0]), qa1 = smem_u32(&s.q[qb1][0][0]);
+            // descriptors of the item's Q tiles; a K stage's is kdesc0 + stage * KSTAGE_DESC
+            const uint64_t qd0 = qdesc0 + (uint64_t)(qb0 * QBUF_DESC);
+            const uint64_t qd1 = qdesc0 + (uint64_t)(qb1 * QBUF_DESC);
             int local = 0;
             auto mma_tile = [&](int kt, bool transposed) {
                 const int stage = it % STAGES;
@@ -446,13 +471,12 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
                     ok = false;
                     return;
                 }
-                const uint32_t ka = smem_u32(&s.k[stage][0][0]);
+                const uint64_t kd = kdesc0 + (uint64_t)(stage * KSTAGE_DESC);
 #pragma unroll
                 for (int gp = 0; gp < NGRP; ++gp) {
                     // which group receives an accumulator for this tile, and from which Q tile
                     const bool mine = itm.nr == 2 ? kt < itm.nt[gp] : (local & 1) == gp;
                     if (!mine) continue;
-                    const uint32_t qaddr = (itm.nr == 2 && gp == 1) ? qa1 : qa0;
                     const int b = acc[gp] & 1;
                     if (!tc::mbar_wait(&s.s_empty[gp][b], ((acc[gp] >> 1) & 1) ^ 1, abort_flag)) {
                         ok = false;
@@ -460,13 +484,11 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
                     }
                     tc::fence_after_sync();
                     const uint32_t d_tmem = tmem + (uint32_t)((gp * 2 + b) * BN);
-#pragma unroll
-                    for (int kk = 0; kk < D / 16; ++kk) {
-                        const uint32_t off = (uint32_t)((kk >> 2) * (BM * 64 * 2) + (kk & 3) * 32);
-                        const uint64_t qd = tc::sdesc_k_sw128(qaddr + off);
-                        const uint64_t kd = tc::sdesc_k_sw128(ka + off);
-                        tc::mma_bf16(d_tmem, transposed ? kd : qd, transposed ? qd : kd, IDESC, kk > 0);
-                    }
+                    const uint64_t qd = (itm.nr == 2 && gp == 1) ? qd1 : qd0;
+                    if (transposed)
+                        mma_kq<D, true>(d_tmem, qd, kd);
+                    else
+                        mma_kq<D, false>(d_tmem, qd, kd);
                     tc::mma_commit(&s.s_full[gp][b]);
                     ++acc[gp];
                 }
