@@ -58,7 +58,8 @@ constexpr int NQB = 2;            // Q tiles in shared memory
 constexpr int NIQ = 2;            // items fetched ahead
 constexpr int GSOFT = 256;        // threads per softmax group (2 warps per lane quarter)
 constexpr int NSOFT = NGRP * GSOFT;
-constexpr int NTHREADS = 64 + NSOFT;
+constexpr int MMA2_WARP = 2 + NSOFT / 32;   // the second MMA issuer, after the softmax warps
+constexpr int NTHREADS = 64 + NSOFT + 32;
 constexpr int TMEM_COLS = 512;    // 2 accumulators x 2 groups x 128 columns
 constexpr int MAXT = kMaxN / BN;  // key tiles per head
 constexpr int MAX_RT = 256;       // row tiles per KV head (G * n_win <= 32768)
@@ -290,11 +291,11 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
             }
         for (int i = 0; i < NQB; ++i) {
             tc::mbar_init(&s.q_full[i], 1);
-            tc::mbar_init(&s.q_empty[i], 1);
+            tc::mbar_init(&s.q_empty[i], 2);    // both MMA issuers
         }
         for (int i = 0; i < NIQ; ++i) {
             tc::mbar_init(&s.it_full[i], 1);
-            tc::mbar_init(&s.it_empty[i], 2);   // the MMA thread and the softmax role
+            tc::mbar_init(&s.it_empty[i], 3);   // the two MMA issuers and the softmax role
         }
         for (int gp = 0; gp < NGRP; ++gp)
             for (int qq = 0; qq < 4; ++qq)
@@ -302,7 +303,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
                     tc::mbar_init(&s.pb_full[gp][qq][i], 1);   // the writer warp of the quarter
                     tc::mbar_init(&s.pb_empty[gp][qq][i], 1);  // the reader warp
                 }
-        tc::mbar_init(&s.mma_done, 1);
+        tc::mbar_init(&s.mma_done, 2);
         tc::fence_mbar_init();
     }
     if (warp == 1) {
@@ -431,8 +432,14 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
             tc::mbar_wait(&s.full[i % STAGES], (i / STAGES) & 1, &s.never);
     }
 
-    // ------------------------------------------------------------ MMA issuer
-    if (warp == 1 && lane == 0) {
+    // ------------------------------------------------------------ MMA issuers
+    // Two threads in different warps issue the MMAs of alternate ring entries.
+    // A thread that uses the outcome of an mbarrier wait stalls until its own
+    // MMAs in flight have drained; with two issuers the other one keeps the
+    // tensor pipe busy meanwhile.  Both walk every entry to keep the
+    // accumulator counters, and issue only for entries of their parity.
+    if ((warp == 1 || warp == MMA2_WARP) && lane == 0) {
+        const int me = warp == 1 ? 0 : 1;
         // shared-memory descriptors, computed once: the start-address field
         // (16-byte units, < 2^14 inside 256 KB) takes plain additions
         const uint64_t kdesc0 = tc::sdesc_k_sw128(smem_u32(&s.k[0][0][0]));
@@ -467,7 +474,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
             int local = 0;
             auto mma_tile = [&](int kt, bool transposed) {
                 const int stage = it % STAGES;
-                if (!tc::mbar_wait(&s.full[stage], (it / STAGES) & 1, abort_flag)) {
+                const bool issue = (it & 1) == me;
+                if (issue && !tc::mbar_wait(&s.full[stage], (it / STAGES) & 1, abort_flag)) {
                     ok = false;
                     return;
                 }
@@ -478,6 +486,10 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
                     const bool mine = itm.nr == 2 ? kt < itm.nt[gp] : (local & 1) == gp;
                     if (!mine) continue;
                     const int b = acc[gp] & 1;
+                    if (!issue) {
+                        ++acc[gp];
+                        continue;
+                    }
                     if (!tc::mbar_wait(&s.s_empty[gp][b], ((acc[gp] >> 1) & 1) ^ 1, abort_flag)) {
                         ok = false;
                         return;
@@ -492,7 +504,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
                     tc::mma_commit(&s.s_full[gp][b]);
                     ++acc[gp];
                 }
-                tc::mma_commit(&s.empty[stage]);
+                if (issue) tc::mma_commit(&s.empty[stage]);
                 ++it;
                 ++local;
             };
@@ -514,7 +526,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
     }
 
     // ------------------------------------------------------------ softmax groups
-    if (warp >= 2) {
+    if (warp >= 2 && warp < MMA2_WARP) {
         const int sid = tid - 64;
         const int quarter = warp & 3;
         const int grp = (warp - 2) >> 3;
