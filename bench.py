@@ -23,6 +23,8 @@ import sys
 import threading
 import time
 
+import numpy as np
+
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
@@ -50,6 +52,10 @@ def parse():
                     help="wall-clock target of the oracle CPU-baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--record-traffic", metavar="CSV",
+                    help="record the DRAM bytes of one kernel launch from `ncu -i REP --page raw "
+                         "--csv` output into profiles/traffic.json (for --stage and --config)")
+    ap.add_argument("--stage", default="score", choices=["score", "budget", "select", "compact"])
     return ap.parse_args()
 
 
@@ -91,14 +97,27 @@ def stage_bytes(wl, ratio):
     }
 
 
-KERNEL_SOURCES = {"score": "score_tc.cu", "budget": "budget.cu", "select": "select.cu",
-                  "compact": "compact.cu"}
+def score_flops(wl):
+    """Algorithmic FLOPs of the score kernel: the logits q.k of every text-query
+    row of every query head against each key it attends to (causal), once."""
+    visible = int((wl.text_pos.astype(np.int64) + 1).sum())
+    return 2 * wl.d * wl.L * wl.H_q * visible
+
+
+# each kernel's source with the headers it includes (a change to any of them
+# invalidates a recorded ncu traffic figure)
+KERNEL_SOURCES = {"score": ("score_tc.cu", "tc05.cuh", "common.cuh"),
+                  "budget": ("budget.cu", "budget.cuh", "common.cuh"),
+                  "select": ("select.cu", "budget.cuh", "common.cuh"),
+                  "compact": ("compact.cu", "common.cuh")}
 
 
 def source_hash(stage):
-    path = os.path.join(ROOT, "paper_2606_03075_gb300", "csrc", KERNEL_SOURCES[stage])
-    with open(path, "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+    h = hashlib.sha256()
+    for name in KERNEL_SOURCES[stage]:
+        with open(os.path.join(ROOT, "paper_2606_03075_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
 
 
 def recorded_traffic(stage, workload):
@@ -110,6 +129,34 @@ def recorded_traffic(stage, workload):
     except (OSError, KeyError, ValueError):
         return None
     return rec["dram_bytes_per_launch"] if rec.get("source_sha") == source_hash(stage) else None
+
+
+_BYTE_UNITS = {"byte": 1, "Kbyte": 1e3, "Mbyte": 1e6, "Gbyte": 1e9, "Tbyte": 1e12}
+
+
+def record_traffic(csv_path, stage, workload):
+    """Write dram__bytes_read.sum + dram__bytes_write.sum of the first kernel in
+    an ncu raw-page CSV export to profiles/traffic.json."""
+    import csv
+    rows = list(csv.reader(open(csv_path)))
+    head, units, vals = rows[0], rows[1], rows[2]
+    total = 0.0
+    for name in ("dram__bytes_read.sum", "dram__bytes_write.sum"):
+        i = head.index(name)
+        total += float(vals[i].replace(",", "")) * _BYTE_UNITS[units[i]]
+    kernel = vals[head.index("Kernel Name")] if "Kernel Name" in head else "?"
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        rec = json.load(open(path))
+    except (OSError, ValueError):
+        rec = {}
+    rec.setdefault(stage, {})[workload] = {
+        "dram_bytes_per_launch": int(round(total)), "source_sha": source_hash(stage),
+        "kernel": kernel.split("(")[0]}
+    with open(path, "w") as f:
+        json.dump(rec, f, indent=1, sort_keys=True)
+        f.write("\n")
+    print(json.dumps(rec[stage][workload]))
 
 
 def measured_peaks():
@@ -275,12 +322,13 @@ def run_reference(args, rank, world):
 # --------------------------------------------------------------------------
 def main():
     args = parse()
+    if args.record_traffic:
+        return record_traffic(args.record_traffic, args.stage, args.config)
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     if args.impl == "reference":
         return run_reference(args, rank, world)
 
-    import numpy as np
     import torch
     import torch.distributed as dist
 
@@ -312,6 +360,7 @@ def main():
                          text_pos=upload(inp["text_pos"]), w=upload(inp["w"])))
     ws = api.new_workspace(desc, dev)
     out = api.alloc_outputs(desc, ratio, dev)
+    launches_per_step = api.tgvkv_evict_launches(desc)
     stream = torch.cuda.current_stream(dev)
 
     def evict(s):
@@ -327,8 +376,9 @@ def main():
     # ---- warm-up, then the timed region (fused path)
     for s in range(args.warmup):
         evict(s)
-    if api.tgvkv_status(ws, stream) != 0:
-        raise RuntimeError("device status bits set during warm-up")
+    bits = api.tgvkv_status(ws, stream)
+    if bits != 0:
+        raise RuntimeError(f"device status bits 0x{bits:x} set during warm-up")
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(args.steps)]
     barrier()
@@ -342,8 +392,9 @@ def main():
         t_wall = time.perf_counter() - t_wall
     step_ms = [a.elapsed_time(b) for a, b in ev]
     region_ms = ev[0][0].elapsed_time(ev[-1][1])
-    if api.tgvkv_status(ws, stream) != 0:
-        raise RuntimeError("device status bits set in the timed region")
+    bits = api.tgvkv_status(ws, stream)
+    if bits != 0:
+        raise RuntimeError(f"device status bits 0x{bits:x} set in the timed region")
     region = torch.tensor([region_ms], device=dev, dtype=torch.float64)
     if world > 1:
         dist.all_reduce(region, op=dist.ReduceOp.MAX)
@@ -422,10 +473,22 @@ def main():
     # ---- roofline of the dominant kernel and of the whole step
     peaks, peak_src = measured_peaks()
     hbm_peak = float(peaks["hbm_gbs"])
+    tensor_peak = float(peaks["bf16_tflops"])
     sb = stage_bytes(wl, ratio)
     dom = max(stages, key=lambda s: stage_ms[s])
-    achieved = sb[dom] / (stage_ms[dom] * 1e-3) / 1e9
     traffic = recorded_traffic(dom, wl.name)
+    # the binding roof: HBM unless the kernel's algorithmic FLOPs take longer
+    # than its bytes at the respective measured peaks (grouped-query shapes)
+    flops = score_flops(wl) if dom == "score" else 0
+    if flops / (tensor_peak * 1e12) > sb[dom] / (hbm_peak * 1e9):
+        roof = {"bound": "tensor", "achieved": flops / (stage_ms[dom] * 1e-3) / 1e12,
+                "peak": tensor_peak, "unit": "TFLOP/s",
+                "peak_source": f"{peak_src} bf16_tflops (MEASURED_PEAKS.json, burst)"}
+    else:
+        roof = {"bound": "hbm", "achieved": sb[dom] / (stage_ms[dom] * 1e-3) / 1e9,
+                "peak": hbm_peak, "unit": "GB/s",
+                "peak_source": f"{peak_src} hbm_gbs (MEASURED_PEAKS.json)"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
     sbytes, rows = step_bytes(wl, ratio)
     step_gbs = sbytes * args.steps * world / (region_ms * 1e-3) / 1e9
 
@@ -447,16 +510,18 @@ def main():
             "hbm_step": {"bytes_per_step": sbytes, "bytes_per_layer": sbytes / wl.L,
                          "gbs": step_gbs, "peak": hbm_peak, "frac": step_gbs / hbm_peak,
                          "definition": "K read once + compacted K/V written, per step"},
-            "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": hbm_peak,
-                         "unit": "GB/s", "frac": achieved / hbm_peak, "traffic": traffic,
-                         "bytes_per_launch": sb[dom], "launch_ms": stage_ms[dom],
-                         "peak_source": f"{peak_src} hbm_gbs (MEASURED_PEAKS.json)"},
+            "roofline": {"bound": roof["bound"], "kernel": dom, "achieved": roof["achieved"],
+                         "peak": roof["peak"], "unit": roof["unit"], "frac": roof["frac"],
+                         "traffic": traffic, "bytes_per_launch": sb[dom],
+                         "flops_per_launch": flops, "launch_ms": stage_ms[dom],
+                         "peak_source": roof["peak_source"]},
             "stage_ms": stage_ms,
+            "fused_tail_ms": statistics.mean(step_ms) - stage_ms["score"],
             "step_ms_median": statistics.median(step_ms),
             "wall_s_timed_region": t_wall,
             "cpu_baseline": cpu,
             "e2e": e2e,
-            "gpu_launches": 4 * args.steps,
+            "gpu_launches": launches_per_step * args.steps,
             "clocks": clocks.summary(),
         }
     if world > 1:

@@ -150,6 +150,15 @@ int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
                 int64_t* offsets, int32_t* idx, uint16_t* k_out, uint16_t* v_out,
                 void* workspace, void* stream);
 
+/* Number of CUDA kernels one tgvkv_evict call launches for this problem
+ * (introspection for callers that budget launches, e.g. inside a captured
+ * graph; the paper has no counterpart): normally 2 (score, then budget +
+ * select + gather fused), 4 when the fused kernel's shared-memory table does
+ * not fit (score, budget, select, compact), one fewer when the problem has no
+ * query rows (the scores are then zero-filled with memsets).  Returns -1 on
+ * bad arguments. */
+int tgvkv_evict_launches(const tgvkv_desc* desc);
+
 /* Zero `workspace` (asynchronously on `stream`).  Needed once after the
  * workspace is allocated: the calls leave their completion counters at zero
  * for the next call.  Zero it again after a call whose tgvkv_status reported

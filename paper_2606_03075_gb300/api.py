@@ -210,5 +210,13 @@ def tgvkv_status(ws: torch.Tensor, stream=None) -> int:
     return rc
 
 
+def tgvkv_evict_launches(desc: Desc) -> int:
+    """Kernels one tgvkv_evict call launches for this problem."""
+    n = _lib.load().tgvkv_evict_launches(ctypes.byref(desc))
+    if n < 0:
+        raise TgvkvError(-1, "tgvkv_evict_launches")
+    return int(n)
+
+
 def default_scale(d: int) -> float:
     return 1.0 / math.sqrt(d)

@@ -265,6 +265,12 @@ int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
     return ok();
 }
 
+int tgvkv_evict_launches(const tgvkv_desc* desc) {
+    Problem p{};
+    if (make_problem(desc, &p) != TGVKV_OK) return -1;
+    return score_launches(p) + budget_select_compact_launches(p);
+}
+
 int tgvkv_workspace_init(const tgvkv_desc* desc, void* workspace, void* stream) {
     Problem p{};
     int rc = make_problem(desc, &p);

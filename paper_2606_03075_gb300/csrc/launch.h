@@ -36,6 +36,10 @@ cudaError_t launch_budget_select_compact(const Problem& p, const float* scores,
                                          long long capacity_rows, uint32_t* status,
                                          cudaStream_t stream);
 
+// Kernels launch_score / launch_budget_select_compact launch for p.
+int score_launches(const Problem& p);
+int budget_select_compact_launches(const Problem& p);
+
 cudaError_t launch_compact(const Problem& p, const uint16_t* k, const uint16_t* v,
                            const int64_t* offsets, const int32_t* idx, uint16_t* k_out,
                            uint16_t* v_out, long long capacity_rows, uint32_t* status,

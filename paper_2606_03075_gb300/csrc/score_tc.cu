@@ -85,6 +85,7 @@ struct PSmem {
     int item_q[NIQ];
     uint32_t tmem_base;
     int abort_flag, never, stop, head_last, cur_item;
+    int issued[NGRP];                        // accumulator uses issued so far, per group
     float tile_mass[NGRP];
 };
 
@@ -239,6 +240,21 @@ __device__ __forceinline__ float colsum_group(const float (&y)[32], const float*
     return (a.x + a.y) + (b.x + b.y);
 }
 
+// Bounded wait until *counter == value (the other MMA issuer has issued the
+// group's previous accumulator use).
+__device__ __forceinline__ bool wait_turn(const int* counter, int value, volatile int* abort) {
+    const volatile int* c = counter;
+    if (*c == value) return true;
+    const long long c0 = clock64();
+    for (uint32_t i = 1;; ++i) {
+        if (*c == value) return true;
+        if ((i & 63u) == 0) {
+            if (*abort) return false;
+            if (clock64() - c0 > tc::kWaitLimitCycles) return false;
+        }
+    }
+}
+
 // A bounded wait whose outcome is the same for every lane of the warp (the
 // tensor-memory loads that follow are warp-collective).
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
@@ -280,6 +296,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
     if (tid == 0) {
         s.abort_flag = 0;
         s.never = 0;
+        for (int gp = 0; gp < NGRP; ++gp) s.issued[gp] = 0;
         for (int i = 0; i < STAGES; ++i) {
             tc::mbar_init(&s.full[i], 1);
             tc::mbar_init(&s.empty[i], 1);
@@ -438,6 +455,11 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
     // MMAs in flight have drained; with two issuers the other one keeps the
     // tensor pipe busy meanwhile.  Both walk every entry to keep the
     // accumulator counters, and issue only for entries of their parity.
+    // A group's accumulator uses are issued strictly in order across the two
+    // threads (s.issued): when a group skips an entry, the buffer a thread
+    // fills changes, and without the ordering one thread could wait on the
+    // release of use u-2 before the other has issued it -- two phases behind,
+    // which a parity wait cannot tell apart from a completed phase.
     if ((warp == 1 || warp == MMA2_WARP) && lane == 0) {
         const int me = warp == 1 ? 0 : 1;
         // shared-memory descriptors, computed once: the start-address field
@@ -490,7 +512,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
                         ++acc[gp];
                         continue;
                     }
-                    if (!tc::mbar_wait(&s.s_empty[gp][b], ((acc[gp] >> 1) & 1) ^ 1, abort_flag)) {
+                    if (!wait_turn(&s.issued[gp], acc[gp], abort_flag) ||
+                        !tc::mbar_wait(&s.s_empty[gp][b], ((acc[gp] >> 1) & 1) ^ 1, abort_flag)) {
                         ok = false;
                         return;
                     }
@@ -503,6 +526,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
                         mma_kq<D, false>(d_tmem, qd, kd);
                     tc::mma_commit(&s.s_full[gp][b]);
                     ++acc[gp];
+                    *reinterpret_cast<volatile int*>(&s.issued[gp]) = acc[gp];
                 }
                 if (issue) tc::mma_commit(&s.empty[stage]);
                 ++it;
@@ -861,6 +885,8 @@ cudaError_t launch_tc(const Problem& p, const uint16_t* q, const uint16_t* k,
 }
 
 }  // namespace
+
+int score_launches(const Problem& p) { return p.R == 0 ? 0 : 1; }
 
 cudaError_t launch_score(const Problem& p, const uint16_t* q, const uint16_t* k,
                          const uint8_t* modality, const int32_t* text_pos, const float* w,

@@ -268,6 +268,11 @@ cudaError_t launch_select(const Problem& p, const float* scores, const int32_t* 
                                         sizeof(uint32_t) * (size_t)p.N_v, stream);
 }
 
+int budget_select_compact_launches(const Problem& p) {
+    const size_t smem = kBudgetBytes + sizeof(uint32_t) * ((size_t)p.N_v + (size_t)p.N);
+    return smem > kFusedSmemLimit ? 3 : 1;
+}
+
 cudaError_t launch_budget_select_compact(const Problem& p, const float* scores,
                                          const float* tvb_stat, long long budget_total,
                                          int32_t* budgets, const uint8_t* modality,

@@ -45,23 +45,21 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Wait for the phase with the given parity.  Gives up (returns false) after
-// ~kWaitLimitNs of wall time, or early once *abort is set by another role.
-constexpr unsigned long long kWaitLimitNs = 1000ull * 1000ull * 1000ull;  // 1 s
-
-__device__ __forceinline__ unsigned long long global_ns() {
-    unsigned long long t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
+// kWaitLimitCycles SM clock cycles (about 1 s at 2 GHz), or early once *abort
+// is set by another role.  The limit is counted on the SM's own cycle counter,
+// which only moves forward: the global nanosecond timer can be re-synchronised
+// by the driver while a kernel runs, and a step backwards would read as an
+// enormous unsigned elapsed time and end a healthy wait.
+constexpr long long kWaitLimitCycles = 2000ll * 1000ll * 1000ll;
 
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
     if (mbar_try_wait(bar, parity)) return true;
-    const unsigned long long t0 = global_ns();
+    const long long c0 = clock64();
     for (uint32_t i = 1;; ++i) {
         if (mbar_try_wait(bar, parity)) return true;
         if ((i & 63u) == 0) {
             if (*abort) return false;
-            if (global_ns() - t0 > kWaitLimitNs) return false;
+            if (clock64() - c0 > kWaitLimitCycles) return false;
         }
     }
 }

@@ -150,6 +150,28 @@ def test_repeat_calls_are_deterministic(api):
         np.testing.assert_array_equal(a[key], b[key], err_msg=key)
 
 
+def test_back_to_back_launches_stay_clean(api):
+    """Many score launches queued back to back (no host synchronisation between
+    them) on the long interleaved-video shape, whose row-tile pairs have
+    different causal ranges, so a group skips ring entries and the two MMA
+    issuers hand accumulator buffers to each other.  Every launch must finish
+    without a timed-out wait and reproduce the first launch bit for bit."""
+    wl = synth.WORKLOADS["video"]
+    inp = synth.generate(wl, seed=0)
+    dev = P.device_inputs(inp)
+    desc = api.desc_for_workload(wl)
+    ws = api.new_workspace(desc)
+    out = api.alloc_outputs(desc, wl.ratios[0])
+    args = (desc, dev["q"], dev["k"], dev["modality"], dev["text_pos"], dev["w"])
+    api.tgvkv_score(*args, out.scores, out.tvb_stat, ws)
+    assert api.tgvkv_status(ws) == 0
+    first = (out.scores.clone(), out.tvb_stat.clone())
+    for _ in range(150):
+        api.tgvkv_score(*args, out.scores, out.tvb_stat, ws)
+    assert api.tgvkv_status(ws) == 0
+    assert torch.equal(out.scores, first[0]) and torch.equal(out.tvb_stat, first[1])
+
+
 # ---------------------------------------------------------------- single steps
 def test_budget_kernel_exact(api):
     """TVB budgets from crafted statistics, including exact ties, zeros and caps."""
