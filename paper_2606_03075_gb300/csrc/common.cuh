@@ -20,17 +20,24 @@ struct Problem {
 // Workspace layout (byte offsets into the caller's buffer).
 struct WsLayout {
     size_t status;      // uint32 status word
-    size_t tickets;     // uint32 [ticket_words]: completion counters (heads, layers), work counter
+    size_t tickets;     // uint32 [ticket_words]: completion counters (heads), kernel counters
     size_t stat_part;   // float [L*H_kv*T]: TV mass of one row tile
     size_t stat_head;   // float [L*H_kv]: TV mass of one KV head
     size_t score_part;  // float [L*H_kv*T*N_v]: scores of one row tile (T > 1)
     size_t total;
 };
 
-// Counters at the start of the workspace: one per KV head, one per layer, then
-// the score kernel's work counter and its done counter.
+// Work items of one KV head in the score kernel: pairs of 128-row tiles
+// (P = ceil(T / 2)) when the head has more than one row tile, else 1.
+__host__ __device__ inline int score_pairs(const Problem& p) {
+    return p.T >= 2 ? (p.T + 1) / 2 : 1;
+}
+
+// Counters at the start of the workspace: one per KV head, then the score
+// kernel's work counter, the count of CTAs that ran out of work, and the count
+// of CTAs that finished.
 __host__ __device__ inline size_t ticket_words(const Problem& p) {
-    return (size_t)p.L * p.H_kv + p.L + 2;
+    return (size_t)p.L * p.H_kv + 3;
 }
 
 constexpr int kMaxN = 32768;     // key positions per head (the per-CTA tile maps)

@@ -2,41 +2,49 @@
 // a persistent, warp-specialised kernel with one CTA per SM.
 //
 // The query rows of one (layer, KV head) -- the G query heads of the group
-// stacked over the n_win text-query rows -- are cut into 128-row tiles.  Each
-// row tile streams the head's 128-key tiles twice, the two passes of
-// Eq. 2 / Eq. 8:
+// stacked over the n_win text-query rows -- form 128-row tiles.  Every row
+// streams the head's keys twice, the two passes of Eq. 2 / Eq. 8:
 //
 //   pass A  S = Q K^T  (TMEM lane = query row): per row an online maximum m_i,
 //           normaliser Z_i and vision mass V_i over every visible key (causal:
 //           key j <= position of row i).
-//   pass B  S^T = K Q^T  (TMEM lane = key) over the tiles that hold vision
+//   pass B  S^T = K Q^T  (TMEM lane = key) over the key tiles that hold vision
 //           keys: per key j the sum over rows of c_i 2^(x_ij - m_i),
 //           c_i = w_i / (G Z_i) -- the text-weighted column sum of Eq. 8 with
 //           the GQA mean folded in.  c_i goes into the exponent,
 //           2^(x_ij - m'_i) with m'_i = m_i - log2 c_i, so a term is one
-//           packed-pair FFMA, one EX2 and one packed FADD, and the column sum
-//           needs no cross-lane reduction.
+//           FFMA, one EX2 and one FADD, and no cross-lane reduction is needed.
 //
-// Delivering K tiles is what bounds this kernel, so every K tile loaded is
-// used for as many query rows as possible: a work item is a PAIR of row tiles
-// of one head (when the head has more than one), and each K tile feeds two
-// MMAs, one per row tile.  A head with a single row tile is one item.
+// The pipeline moves in steps; a step fills one of two 256-column fp32 TMEM
+// accumulators, and all 16 softmax warps consume every step.  What a step
+// holds depends on the shape of the work item:
 //
-// Roles: warp 0 fetches items from a global counter (longest items first) and
-// issues TMA loads -- the item's Q tiles, then every K tile of both passes
-// through a 4-stage ring, running ahead into the next item; warp 1 owns the
-// SM's 512 TMEM columns (two 128-column fp32 accumulators per softmax group)
-// and one of its lanes issues the MMAs; warps 2-17 form two softmax groups.
-// With a row-tile pair, group g owns row tile g; with a single row tile the
-// groups take alternate K tiles.  In a group, two warps per TMEM lane quarter
-// split a tile's 128 columns.  Every wait is bounded (1 s); a timeout sets
-// TGVKV_STATUS_TIMEOUT and the CTA unwinds.
+//   pair    (a head with 2+ row tiles; an item is two row tiles of one head)
+//           one K tile x both row tiles.  Pass A: columns [128r, 128r+128) =
+//           Q_r K^T.  Pass B: one N = 256 product K [Q_0; Q_1]^T.  Each K tile
+//           is read once for 256 query rows.
+//   single  (one row tile of more than 64 rows) two K tiles x the row tile.
+//   packed  (one row tile of at most 64 rows) TWO heads share the 128 lanes:
+//           head h's rows live in lane quarters 2h and 2h+1, and a step holds
+//           one K tile of each head; columns [128h, 128h+128) are
+//           [Q_0; Q_1] K_h^T, of which only head h's lanes are read (pass A),
+//           and K_h [Q_0; Q_1]^T, of which only head h's columns are read
+//           (pass B).  Every lane and every softmax thread does useful work.
 //
-// Query rows are spread evenly over the four lane quarters (row q*rpg + i ->
-// lane 32q + i) so that all softmax warps share the work when a row tile has
-// fewer than 128 rows.  Row tiles of a head write partial score rows; the last
-// one to finish adds them in tile order, and the last head of a layer adds the
-// TV masses in head order, so the results do not depend on the schedule.
+// Roles: warp 0 fetches items from a global counter (longest first) and issues
+// TMA loads -- an item's Q rows, then every K tile of both passes through a
+// 4-stage ring; warps 1 and 18 issue the MMAs of alternate steps (a thread
+// that waits on an mbarrier lets its own MMA queue drain, so two issuers keep
+// the tensor pipe busy; step k always uses accumulator k & 1, so each issuer
+// owns one accumulator); warp 1 also owns the 512 TMEM columns; warps 2-17 run
+// the softmax, four per TMEM lane quarter.  Every wait is bounded (about 1 s
+// of SM cycles); a timeout sets TGVKV_STATUS_TIMEOUT and the CTA unwinds.
+//
+// Results do not depend on the schedule: every key's pass-B sum is two
+// partial sums added onto zero (the same in either order); the row tiles of a
+// head write partial score rows that the last pair to finish adds in tile
+// order; and the last CTA to finish adds the per-head TV masses of each layer
+// in head order.
 #include <cudaTypedefs.h>
 #include <limits.h>
 #include <math.h>
@@ -51,108 +59,144 @@ namespace tgvkv {
 namespace {
 
 constexpr int BM = 128;           // query rows per row tile = TMEM lanes
-constexpr int BN = 128;           // keys per tile
+constexpr int BN = 128;           // keys per K tile
 constexpr int STAGES = 4;         // K tiles in flight
-constexpr int NGRP = 2;           // softmax groups
-constexpr int NQB = 2;            // Q tiles in shared memory
 constexpr int NIQ = 2;            // items fetched ahead
-constexpr int GSOFT = 256;        // threads per softmax group (2 warps per lane quarter)
-constexpr int NSOFT = NGRP * GSOFT;
-constexpr int MMA2_WARP = 2 + NSOFT / 32;   // the second MMA issuer, after the softmax warps
-constexpr int NTHREADS = 64 + NSOFT + 32;
-constexpr int TMEM_COLS = 512;    // 2 accumulators x 2 groups x 128 columns
+constexpr int NSW = 16;           // softmax warps (4 per TMEM lane quarter)
+constexpr int NSOFT = NSW * 32;
+constexpr int MMA2_WARP = 2 + NSW;
+constexpr int NTHREADS = (NSW + 3) * 32;
+constexpr int SCOLS = 256;        // accumulator columns per step
+constexpr int TMEM_COLS = 2 * SCOLS;
 constexpr int MAXT = kMaxN / BN;  // key tiles per head
 constexpr int MAX_RT = 256;       // row tiles per KV head (G * n_win <= 32768)
-constexpr uint32_t IDESC = tc::idesc_bf16(128, 128);
+constexpr uint32_t IDESC128 = tc::idesc_bf16(128, 128);
+constexpr uint32_t IDESC256 = tc::idesc_bf16(128, 256);
+constexpr uint32_t IDESC64 = tc::idesc_bf16(128, 64);
+
+enum { MODE_PAIR = 0, MODE_SINGLE = 1, MODE_PACKED = 2 };
 
 template <int D>
 struct PSmem {
-    uint16_t q[NQB][D / 64][BM * 64];        // Q tiles, one 128-byte-swizzled half per 64 dims
+    uint16_t q[D / 64][2][BM * 64];          // two Q slots; per 64 dims, 128-byte-swizzled rows
     uint16_t k[STAGES][D / 64][BN * 64];     // K ring
     uint64_t full[STAGES], empty[STAGES];
-    uint64_t s_full[NGRP][2], s_empty[NGRP][2];
-    uint64_t q_full[NQB], q_empty[NQB], mma_done;
+    uint64_t s_full[2], s_empty[2];
+    uint64_t q_full[2], q_empty[2], mma_done;
     uint64_t it_full[NIQ], it_empty[NIQ];
-    uint64_t pb_full[NGRP][4][2], pb_empty[NGRP][4][2];  // pass-B hand-off per group and quarter
     uint32_t vmask[MAXT][4];                 // vision bit of each key of each tile
     int vis_before[MAXT + 1];                // vision keys before each tile
+    int vq[MAXT][4];                         // vision keys before each 32-key word
     int rt_max[MAX_RT], rt_min[MAX_RT];      // per row tile: max / min query position
-    alignas(16) int row_pos[NGRP][BM];       // per group and TMEM lane: row position, -1 = none
-    alignas(16) float row_nmp[NGRP][BM];     // -(m_i - log2 c_i); -inf = no row
-    float row_w[NGRP][BM], row_mass[NGRP][BM];
-    float part_m[NGRP * 2][BM], part_z[NGRP * 2][BM], part_v[NGRP * 2][BM];
-    float pbuf[NGRP][2][BM];
+    alignas(16) int row_pos[2][BM];          // per row slot and TMEM lane: position, -1 = none
+    alignas(16) float row_nmp[2][BM];        // -(m_i - log2 c_i); -inf = no row
+    float row_w[2][BM], row_mass[2][BM];
+    float part_m[4][BM], part_z[4][BM], part_v[4][BM];
     int item_q[NIQ];
     uint32_t tmem_base;
-    int abort_flag, never, stop, head_last, cur_item;
-    int issued[NGRP];                        // accumulator uses issued so far, per group
-    float tile_mass[NGRP];
+    int abort_flag, never, stop, head_last, cur_item, cta_last;
+    float tile_mass[2];
 };
 
-// One work item: one or two row tiles of one (layer, KV head).
+// One work item.  "part" 0/1 is a row tile (pair) or a head (packed); a single
+// item has part 0 only.
 struct Item {
-    int lh, l, g, nr, ntmax;
-    int t[2], nt[2], rows[2], rpg[2], minp[2];
-    // element r (0 or 1) without a run-time array index
+    int lh[2], l[2];          // (layer, KV head) of each part; lh[1] < 0: absent
+    int qy[2];                // first global Q row of each part's rows
+    int rows[2], rpg[2];      // rows of each part, and rows per 32-lane group
+    int nt[2], minp[2];       // pass-A key tiles and least query position of each part
+    int ntmax, nparts, pidx;  // pidx: which pair of the head (pair items)
     __device__ __forceinline__ static int pick(const int (&a)[2], int r) { return r ? a[1] : a[0]; }
 };
-
-template <int D>
-__device__ __forceinline__ Item item_info(const Problem& p, const PSmem<D>& s, int id, int npair,
-                                          bool pair) {
-    Item it;
-    it.lh = id / npair;
-    const int tp = npair - 1 - id % npair;   // later row tiles (longer causal range) first
-    it.l = it.lh / p.H_kv;
-    it.g = it.lh % p.H_kv;
-    it.t[0] = pair ? 2 * tp : tp;
-    it.t[1] = (pair && 2 * tp + 1 < p.T) ? 2 * tp + 1 : -1;
-    it.nr = it.t[1] >= 0 ? 2 : 1;
-    it.ntmax = 0;
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-        const int t = it.t[r] >= 0 ? it.t[r] : it.t[0];
-        it.rows[r] = min(BM, p.R - t * BM);
-        it.rpg[r] = (it.rows[r] + 3) >> 2;
-        it.nt[r] = (s.rt_max[t] + BN) / BN;
-        it.minp[r] = s.rt_min[t];
-    }
-    it.ntmax = it.nr == 2 ? max(it.nt[0], it.nt[1]) : it.nt[0];
-    return it;
-}
-
-// One 128 x 128 x D product into the accumulator at d_tmem: D/16 MMAs whose
-// operand descriptors differ from the tile's base descriptors by constants
-// (K offset of 32 bytes inside a 128-byte swizzle atom, 16 KB per 64 dims).
-// Pass A: S = Q K^T (TRANS = false); pass B: S^T = K Q^T.
-template <int D, bool TRANS>
-__device__ __forceinline__ void mma_kq(uint32_t d_tmem, uint64_t qd, uint64_t kd) {
-#pragma unroll
-    for (int kk = 0; kk < D / 16; ++kk) {
-        const uint64_t o = (uint64_t)((kk >> 2) * (BM * 64 * 2 / 16) + (kk & 3) * 2);
-        const uint64_t a = TRANS ? kd + o : qd + o, b = TRANS ? qd + o : kd + o;
-        if (kk == 0)
-            tc::mma_bf16_c<0>(d_tmem, a, b, IDESC);
-        else
-            tc::mma_bf16_c<1>(d_tmem, a, b, IDESC);
-    }
-}
 
 __device__ __forceinline__ int next_vis_tile(const int* vis_before, int kt, int n_tiles) {
     while (kt < n_tiles && vis_before[kt + 1] == vis_before[kt]) ++kt;
     return kt;
 }
 
-__device__ __forceinline__ float max32(const float (&x)[32]) {
-    float a = fmaxf(x[0], x[1]), b = fmaxf(x[2], x[3]), c = fmaxf(x[4], x[5]), d = fmaxf(x[6], x[7]);
+template <int D>
+__device__ __forceinline__ Item item_info(const Problem& p, const PSmem<D>& s, int mode, int id) {
+    Item it;
+    const int LH = p.L * p.H_kv;
+    it.pidx = 0;
+    if (mode == MODE_PAIR) {
+        const int npair = score_pairs(p);
+        const int lh = id / npair;
+        const int tp = npair - 1 - id % npair;   // later row tiles (longer causal range) first
+        it.pidx = tp;
+        const int t0 = 2 * tp, t1 = 2 * tp + 1 < p.T ? 2 * tp + 1 : -1;
+        it.nparts = t1 >= 0 ? 2 : 1;
 #pragma unroll
-    for (int i = 8; i < 32; i += 4) {
-        a = fmaxf(a, x[i]);
-        b = fmaxf(b, x[i + 1]);
-        c = fmaxf(c, x[i + 2]);
-        d = fmaxf(d, x[i + 3]);
+        for (int r = 0; r < 2; ++r) {
+            const int t = r == 0 ? t0 : (t1 >= 0 ? t1 : t0);
+            it.lh[r] = (r == 0 || t1 >= 0) ? lh : -1;
+            it.l[r] = lh / p.H_kv;
+            it.qy[r] = (it.l[r] * p.H_q + (lh % p.H_kv) * p.G) * p.n_win + t * BM;
+            it.rows[r] = min(BM, p.R - t * BM);
+            it.rpg[r] = (it.rows[r] + 3) >> 2;
+            it.nt[r] = (s.rt_max[t] + BN) / BN;
+            it.minp[r] = s.rt_min[t];
+        }
+    } else {
+        const bool packed = mode == MODE_PACKED;
+        it.nparts = 1;
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+            const int lh = packed ? 2 * id + r : id;
+            it.lh[r] = (r == 0 || (packed && lh < LH)) ? lh : -1;
+            if (it.lh[r] >= 0 && r == 1) it.nparts = 2;
+            const int lhv = it.lh[r] >= 0 ? lh : id;
+            it.l[r] = lhv / p.H_kv;
+            it.qy[r] = (it.l[r] * p.H_q + (lhv % p.H_kv) * p.G) * p.n_win;
+            it.rows[r] = p.R;
+            it.rpg[r] = packed ? (p.R + 1) >> 1 : (p.R + 3) >> 2;
+            it.nt[r] = (s.rt_max[0] + BN) / BN;
+            it.minp[r] = s.rt_min[0];
+        }
     }
-    return fmaxf(fmaxf(a, b), fmaxf(c, d));
+    it.ntmax = it.nparts == 2 ? max(it.nt[0], it.nt[1]) : it.nt[0];
+    return it;
+}
+
+// Key tiles of the next step of a pass (0 = A, 1 = B); false at the end.
+// kt[1] is the second tile of a single step or the second head's tile of a
+// packed step (-1: none); pair steps use kt[0] for both row tiles.
+__device__ __forceinline__ bool next_step(const Item& it, int mode, int pass, int& cur,
+                                          const int* vis_before, int (&kt)[2]) {
+    int c = pass == 0 ? cur : next_vis_tile(vis_before, cur, it.ntmax);
+    if (c >= it.ntmax) return false;
+    kt[0] = c;
+    cur = c + 1;
+    kt[1] = -1;
+    if (mode == MODE_SINGLE) {
+        const int c2 = pass == 0 ? cur : next_vis_tile(vis_before, cur, it.ntmax);
+        if (c2 < it.ntmax) {
+            kt[1] = c2;
+            cur = c2 + 1;
+        }
+    } else if (mode == MODE_PACKED && it.lh[1] >= 0) {
+        kt[1] = c;
+    }
+    return true;
+}
+
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+    float r;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+    return r;
+}
+
+__device__ __forceinline__ float max32(const float (&x)[32]) {
+    float a = fmax3(x[0], x[1], x[2]), b = fmax3(x[3], x[4], x[5]), c = fmax3(x[6], x[7], x[8]);
+    float d = fmax3(x[9], x[10], x[11]), e = fmax3(x[12], x[13], x[14]);
+    float f = fmax3(x[15], x[16], x[17]), g = fmax3(x[18], x[19], x[20]);
+    float h = fmax3(x[21], x[22], x[23]), i = fmax3(x[24], x[25], x[26]);
+    float j = fmax3(x[27], x[28], x[29]), k = fmaxf(x[30], x[31]);
+    a = fmax3(a, b, c);
+    d = fmax3(d, e, f);
+    g = fmax3(g, h, i);
+    j = fmaxf(j, k);
+    return fmaxf(fmax3(a, d, g), j);
 }
 
 __device__ __forceinline__ float max32_masked(const float (&x)[32], int lim) {
@@ -210,6 +254,27 @@ __device__ __forceinline__ void exp_word(const float (&x)[32], float sl2, float 
     }
 }
 
+// Online statistics of one row over one 32-key word: columns 0..lim visible.
+__device__ __forceinline__ void row_word(const float (&x)[32], float sl2, int lim, uint32_t vm,
+                                         float& m, float& z, float& v) {
+    if (lim < 0) return;
+    if (lim >= 31) {
+        const float m_new = fmaxf(m, max32(x) * sl2);
+        const float alpha = fast_exp2(m - m_new);
+        z *= alpha;
+        v *= alpha;
+        exp_word<false>(x, sl2, -m_new, 31, vm, z, v);
+        m = m_new;
+    } else {
+        const float m_new = fmaxf(m, max32_masked(x, lim) * sl2);
+        const float alpha = fast_exp2(m - m_new);
+        z *= alpha;
+        v *= alpha;
+        exp_word<true>(x, sl2, -m_new, lim, vm, z, v);
+        m = m_new;
+    }
+}
+
 // Sum over the valid rows of one 32-row group of 2^(y_i sl2 + nmp_i), with the
 // causal mask j <= pos_i unless every row sees key j.  FULL: all 32 rows exist.
 template <bool FULL>
@@ -240,21 +305,6 @@ __device__ __forceinline__ float colsum_group(const float (&y)[32], const float*
     return (a.x + a.y) + (b.x + b.y);
 }
 
-// Bounded wait until *counter == value (the other MMA issuer has issued the
-// group's previous accumulator use).
-__device__ __forceinline__ bool wait_turn(const int* counter, int value, volatile int* abort) {
-    const volatile int* c = counter;
-    if (*c == value) return true;
-    const long long c0 = clock64();
-    for (uint32_t i = 1;; ++i) {
-        if (*c == value) return true;
-        if ((i & 63u) == 0) {
-            if (*abort) return false;
-            if (clock64() - c0 > tc::kWaitLimitCycles) return false;
-        }
-    }
-}
-
 // A bounded wait whose outcome is the same for every lane of the warp (the
 // tensor-memory loads that follow are warp-collective).
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
@@ -262,10 +312,36 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volati
     return __all_sync(~0u, got);
 }
 
+// D/16 MMAs of one 128-row x N-column product, K = D in steps of 16.  a / b
+// are the descriptors of the operands' first 64-dim half; a 64-dim half of an
+// operand lies a_half / b_half 16-byte units further (the 32-byte K step
+// inside a 128-byte swizzle atom is 2 units).
 template <int D>
+__device__ __forceinline__ void mma_block(uint32_t d_tmem, uint64_t a, uint32_t a_half, uint64_t b,
+                                          uint32_t b_half, uint32_t idesc) {
+#pragma unroll
+    for (int kk = 0; kk < D / 16; ++kk) {
+        const uint64_t ka = a + (uint64_t)((kk >> 2) * a_half + (kk & 3) * 2);
+        const uint64_t kb = b + (uint64_t)((kk >> 2) * b_half + (kk & 3) * 2);
+        if (kk == 0)
+            tc::mma_bf16_c<0>(d_tmem, ka, kb, idesc);
+        else
+            tc::mma_bf16_c<1>(d_tmem, ka, kb, idesc);
+    }
+}
+
+// Release this warp's claim on a step accumulator (after its tensor-memory
+// loads have completed).
+__device__ __forceinline__ void release_acc(uint64_t* bar, int lane) {
+    tc::fence_before_sync();
+    __syncwarp();
+    if (lane == 0) tc::mbar_arrive(bar);
+}
+
+template <int D, int MODE>
 __global__ void __launch_bounds__(NTHREADS, 1)
 score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
-                Problem p, const uint8_t* __restrict__ modality,
+                Problem p, int n_items, const uint8_t* __restrict__ modality,
                 const int32_t* __restrict__ text_pos, const float* __restrict__ w,
                 float* __restrict__ scores, float* __restrict__ tvb_stat,
                 float* __restrict__ score_part, float* __restrict__ stat_part,
@@ -274,16 +350,19 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
     extern __shared__ unsigned char smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     PSmem<D>& s = *reinterpret_cast<PSmem<D>*>(smem_raw + (((raw + 1023u) & ~1023u) - raw));
-    constexpr uint32_t TILE_BYTES = (D / 64) * BN * 128;   // one K tile = one Q tile
+    constexpr uint32_t KTILE_BYTES = (D / 64) * BN * 128;
+    constexpr uint32_t QBOX_BYTES = 32 * 128;            // 32 rows x 64 dims
+    constexpr uint32_t K_HALF = BN * 64 * 2 / 16;        // 64-dim half of a K tile, 16-byte units
+    constexpr uint32_t Q_HALF = 2 * BM * 64 * 2 / 16;    // 64-dim half of the Q slots
+    constexpr uint32_t Q_SLOT = BM * 64 * 2 / 16;
 
+    constexpr int mode = MODE;   // the item shape, fixed per launch
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int T = p.T;
-    const bool pair = T >= 2;
-    const int npair = pair ? (T + 1) / 2 : 1;
-    const int n_items = p.L * p.H_kv * npair;
     const float sl2 = p.scale_log2;
-    uint32_t* work_counter = tickets + p.L * p.H_kv + p.L;
+    const int LH = p.L * p.H_kv;
+    uint32_t* work_counter = tickets + LH;
     uint32_t* done_counter = work_counter + 1;
+    uint32_t* exit_counter = work_counter + 2;
 
     // ------------------------------------------------------------ prologue
     if (blockIdx.x == 0) {
@@ -296,30 +375,20 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
     if (tid == 0) {
         s.abort_flag = 0;
         s.never = 0;
-        for (int gp = 0; gp < NGRP; ++gp) s.issued[gp] = 0;
         for (int i = 0; i < STAGES; ++i) {
             tc::mbar_init(&s.full[i], 1);
             tc::mbar_init(&s.empty[i], 1);
         }
-        for (int gp = 0; gp < NGRP; ++gp)
-            for (int i = 0; i < 2; ++i) {
-                tc::mbar_init(&s.s_full[gp][i], 1);
-                tc::mbar_init(&s.s_empty[gp][i], GSOFT / 32);   // one arrival per warp of the group
-            }
-        for (int i = 0; i < NQB; ++i) {
+        for (int i = 0; i < 2; ++i) {
+            tc::mbar_init(&s.s_full[i], 1);
+            tc::mbar_init(&s.s_empty[i], NSW);   // one arrival per softmax warp
             tc::mbar_init(&s.q_full[i], 1);
-            tc::mbar_init(&s.q_empty[i], 2);    // both MMA issuers
+            tc::mbar_init(&s.q_empty[i], 2);     // both MMA issuers
         }
         for (int i = 0; i < NIQ; ++i) {
             tc::mbar_init(&s.it_full[i], 1);
-            tc::mbar_init(&s.it_empty[i], 3);   // the two MMA issuers and the softmax role
+            tc::mbar_init(&s.it_empty[i], 3);    // the two MMA issuers and the softmax role
         }
-        for (int gp = 0; gp < NGRP; ++gp)
-            for (int qq = 0; qq < 4; ++qq)
-                for (int i = 0; i < 2; ++i) {
-                    tc::mbar_init(&s.pb_full[gp][qq][i], 1);   // the writer warp of the quarter
-                    tc::mbar_init(&s.pb_empty[gp][qq][i], 1);  // the reader warp
-                }
         tc::mbar_init(&s.mma_done, 2);
         tc::fence_mbar_init();
     }
@@ -334,12 +403,15 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
         for (int wd = 0; wd < 4; ++wd) {
             const int j = kt * BN + wd * 32 + lane;
             const unsigned m = __ballot_sync(~0u, j < p.N && modality[j] != 0);
-            if (lane == 0) s.vmask[kt][wd] = m;
+            if (lane == 0) {
+                s.vmask[kt][wd] = m;
+                s.vq[kt][wd] = cnt;              // within the tile, for now
+            }
             cnt += __popc(m);
         }
         if (lane == 0) s.vis_before[kt] = cnt;
     }
-    for (int t = tid; t < T; t += NTHREADS) {
+    for (int t = tid; t < p.T; t += NTHREADS) {
         s.rt_max[t] = -1;
         s.rt_min[t] = INT_MAX;
     }
@@ -354,6 +426,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
         }
     }
     if (warp == 0) {
+        // exclusive scan of the per-tile vision counts
         const int per = (n_tiles_all + 31) / 32;
         const int b = lane * per, e = min(b + per, n_tiles_all);
         int sum = 0;
@@ -377,6 +450,10 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
         }
     }
     __syncthreads();
+    for (int kt = tid; kt < n_tiles_all; kt += NTHREADS)
+#pragma unroll
+        for (int wd = 0; wd < 4; ++wd) s.vq[kt][wd] += s.vis_before[kt];
+    __syncthreads();
     const uint32_t tmem = s.tmem_base;
     volatile int* abort_flag = &s.abort_flag;
 
@@ -384,7 +461,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
     if (warp == 0 && lane == 0) {
         tc::tma_prefetch_desc(&tmap_q);
         tc::tma_prefetch_desc(&tmap_k);
-        int it = 0, qn = 0;
+        int it = 0;
+        int qn[2] = {0, 0};
         bool ok = true;
         for (int n = 0; ok; ++n) {
             // fetch the next item (or the end mark) for every role of this CTA
@@ -397,69 +475,74 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
             s.item_q[slot] = id < n_items ? id : -1;
             tc::mbar_arrive(&s.it_full[slot]);
             if (id >= n_items) {
-                // the last CTA to run out of work re-arms the counters for the next launch
+                // the last CTA to run out of work re-arms the counter for the next launch
                 if (atomicAdd(done_counter, 1u) == gridDim.x - 1) {
                     *work_counter = 0u;
                     *done_counter = 0u;
                 }
                 break;
             }
-            const Item itm = item_info(p, s, id, npair, pair);
-            for (int r = 0; r < itm.nr; ++r, ++qn) {
-                const int qb = qn % NQB;
-                if (!tc::mbar_wait(&s.q_empty[qb], ((qn / NQB) & 1) ^ 1, abort_flag)) {
+            const Item itm = item_info(p, s, mode, id);
+            // Q rows: pair items fill both slots (row tile r -> slot r); single
+            // and packed items alternate slots.  Four boxes of 32 rows per slot,
+            // box g landing in TMEM lanes 32g..32g+31.
+            const int nslot = mode == MODE_PAIR ? itm.nparts : 1;
+            for (int r = 0; r < nslot; ++r) {
+                const int qs = mode == MODE_PAIR ? r : (n & 1);
+                if (!tc::mbar_wait(&s.q_empty[qs], (qn[qs] & 1) ^ 1, abort_flag)) {
                     ok = false;
                     break;
                 }
-                const int qy = (itm.l * p.H_q + itm.g * p.G) * p.n_win + Item::pick(itm.t, r) * BM;
-                tc::mbar_arrive_expect_tx(&s.q_full[qb], TILE_BYTES);
+                ++qn[qs];
+                tc::mbar_arrive_expect_tx(&s.q_full[qs], 4 * (D / 64) * QBOX_BYTES);
 #pragma unroll
-                for (int qg = 0; qg < 4; ++qg)
+                for (int qg = 0; qg < 4; ++qg) {
+                    int y;
+                    if (mode == MODE_PACKED) {
+                        const int h = (qg >> 1) < itm.nparts ? (qg >> 1) : 0;
+                        y = Item::pick(itm.qy, h) + (qg & 1) * itm.rpg[0];
+                    } else {
+                        y = Item::pick(itm.qy, r) + qg * Item::pick(itm.rpg, r);
+                    }
 #pragma unroll
                     for (int h = 0; h < D / 64; ++h)
-                        tc::tma_load_2d(&s.q[qb][h][qg * 32 * 64], &tmap_q, h * 64,
-                                        qy + qg * Item::pick(itm.rpg, r), &s.q_full[qb]);
+                        tc::tma_load_2d(&s.q[h][qs][qg * 32 * 64], &tmap_q, h * 64, y, &s.q_full[qs]);
+                }
             }
-            auto issue = [&](int kt) {
+            auto load = [&](int lh, int kt) {
                 const int stage = it % STAGES;
                 if (!tc::mbar_wait(&s.empty[stage], ((it / STAGES) & 1) ^ 1, abort_flag)) {
                     ok = false;
                     return;
                 }
-                tc::mbar_arrive_expect_tx(&s.full[stage], TILE_BYTES);
+                tc::mbar_arrive_expect_tx(&s.full[stage], KTILE_BYTES);
 #pragma unroll
                 for (int h = 0; h < D / 64; ++h)
-                    tc::tma_load_2d(&s.k[stage][h][0], &tmap_k, h * 64, itm.lh * p.N + kt * BN,
+                    tc::tma_load_2d(&s.k[stage][h][0], &tmap_k, h * 64, lh * p.N + kt * BN,
                                     &s.full[stage]);
                 ++it;
             };
-            for (int kt = 0; ok && kt < itm.ntmax; ++kt) issue(kt);
-            for (int kt = next_vis_tile(s.vis_before, 0, itm.ntmax); ok && kt < itm.ntmax;
-                 kt = next_vis_tile(s.vis_before, kt + 1, itm.ntmax))
-                issue(kt);
+            for (int pass = 0; ok && pass < 2; ++pass) {
+                int cur = 0, kt[2];
+                while (ok && next_step(itm, mode, pass, cur, s.vis_before, kt)) {
+                    load(itm.lh[0], kt[0]);
+                    if (ok && kt[1] >= 0) load(mode == MODE_PACKED ? itm.lh[1] : itm.lh[0], kt[1]);
+                }
+            }
         }
         if (!ok) {
             s.abort_flag = 1;
             raise_status(status, TGVKV_STATUS_TIMEOUT);
         }
         // every copy this CTA issued has landed before it may exit
-        for (int i = max(0, qn - NQB); i < qn; ++i)
-            tc::mbar_wait(&s.q_full[i % NQB], (i / NQB) & 1, &s.never);
+        for (int qs = 0; qs < 2; ++qs)
+            if (qn[qs] > 0) tc::mbar_wait(&s.q_full[qs], (qn[qs] - 1) & 1, &s.never);
         for (int i = max(0, it - STAGES); i < it; ++i)
             tc::mbar_wait(&s.full[i % STAGES], (i / STAGES) & 1, &s.never);
     }
 
     // ------------------------------------------------------------ MMA issuers
-    // Two threads in different warps issue the MMAs of alternate ring entries.
-    // A thread that uses the outcome of an mbarrier wait stalls until its own
-    // MMAs in flight have drained; with two issuers the other one keeps the
-    // tensor pipe busy meanwhile.  Both walk every entry to keep the
-    // accumulator counters, and issue only for entries of their parity.
-    // A group's accumulator uses are issued strictly in order across the two
-    // threads (s.issued): when a group skips an entry, the buffer a thread
-    // fills changes, and without the ordering one thread could wait on the
-    // release of use u-2 before the other has issued it -- two phases behind,
-    // which a parity wait cannot tell apart from a completed phase.
+    // Step k goes to issuer k & 1 and accumulator k & 1.
     if ((warp == 1 || warp == MMA2_WARP) && lane == 0) {
         const int me = warp == 1 ? 0 : 1;
         // shared-memory descriptors, computed once: the start-address field
@@ -467,9 +550,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
         const uint64_t kdesc0 = tc::sdesc_k_sw128(smem_u32(&s.k[0][0][0]));
         const uint64_t qdesc0 = tc::sdesc_k_sw128(smem_u32(&s.q[0][0][0]));
         constexpr uint32_t KSTAGE_DESC = (uint32_t)(sizeof(s.k[0]) >> 4);
-        constexpr uint32_t QBUF_DESC = (uint32_t)(sizeof(s.q[0]) >> 4);
-        int it = 0, qn = 0;
-        int acc[NGRP] = {0, 0};
+        int it = 0, step = 0;
+        int qn[2] = {0, 0};
         bool ok = true;
         for (int n = 0; ok; ++n) {
             const int slot = n % NIQ;
@@ -480,65 +562,70 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
             const int id = s.item_q[slot];
             tc::mbar_arrive(&s.it_empty[slot]);
             if (id < 0) break;
-            const Item itm = item_info(p, s, id, npair, pair);
-            // Q tiles of this item: slot qb0 (and qb1 for a pair)
-            const int qb0 = qn % NQB, qb1 = (qn + 1) % NQB;
-            for (int r = 0; r < itm.nr; ++r, ++qn) {
-                if (!tc::mbar_wait(&s.q_full[qn % NQB], (qn / NQB) & 1, abort_flag)) {
+            const Item itm = item_info(p, s, mode, id);
+            const int nslot = mode == MODE_PAIR ? itm.nparts : 1;
+            const int qs0 = mode == MODE_PAIR ? 0 : (n & 1);
+            for (int r = 0; r < nslot; ++r) {
+                const int qs = mode == MODE_PAIR ? r : qs0;
+                if (!tc::mbar_wait(&s.q_full[qs], qn[qs] & 1, abort_flag)) {
                     ok = false;
                     break;
                 }
+                ++qn[qs];
             }
             if (!ok) break;
-            // descriptors of the item's Q tiles; a K stage's is kdesc0 + stage * KSTAGE_DESC
-            const uint64_t qd0 = qdesc0 + (uint64_t)(qb0 * QBUF_DESC);
-            const uint64_t qd1 = qdesc0 + (uint64_t)(qb1 * QBUF_DESC);
-            int local = 0;
-            auto mma_tile = [&](int kt, bool transposed) {
-                const int stage = it % STAGES;
-                const bool issue = (it & 1) == me;
-                if (issue && !tc::mbar_wait(&s.full[stage], (it / STAGES) & 1, abort_flag)) {
-                    ok = false;
-                    return;
-                }
-                const uint64_t kd = kdesc0 + (uint64_t)(stage * KSTAGE_DESC);
-#pragma unroll
-                for (int gp = 0; gp < NGRP; ++gp) {
-                    // which group receives an accumulator for this tile, and from which Q tile
-                    const bool mine = itm.nr == 2 ? kt < itm.nt[gp] : (local & 1) == gp;
-                    if (!mine) continue;
-                    const int b = acc[gp] & 1;
-                    if (!issue) {
-                        ++acc[gp];
-                        continue;
+            const uint64_t qd = qdesc0 + (uint64_t)(qs0 * Q_SLOT);
+            for (int pass = 0; ok && pass < 2; ++pass) {
+                int cur = 0, kt[2];
+                while (ok && next_step(itm, mode, pass, cur, s.vis_before, kt)) {
+                    const int nst = kt[1] >= 0 && mode != MODE_PAIR ? 2 : 1;
+                    if ((step & 1) == me) {
+                        const int b = step & 1;
+                        bool got = tc::mbar_wait(&s.full[it % STAGES], (it / STAGES) & 1, abort_flag);
+                        if (got && nst == 2)
+                            got = tc::mbar_wait(&s.full[(it + 1) % STAGES], ((it + 1) / STAGES) & 1,
+                                                abort_flag);
+                        if (got) got = tc::mbar_wait(&s.s_empty[b], ((step >> 1) & 1) ^ 1, abort_flag);
+                        if (!got) {
+                            ok = false;
+                            break;
+                        }
+                        tc::fence_after_sync();
+                        const uint32_t d = tmem + (uint32_t)(b * SCOLS);
+                        const uint64_t k0 = kdesc0 + (uint64_t)((it % STAGES) * KSTAGE_DESC);
+                        const uint64_t k1 = kdesc0 + (uint64_t)(((it + 1) % STAGES) * KSTAGE_DESC);
+                        if (mode == MODE_PAIR) {
+                            if (pass == 0) {
+                                if (kt[0] < itm.nt[0])
+                                    mma_block<D>(d, qd, Q_HALF, k0, K_HALF, IDESC128);
+                                if (itm.nparts == 2 && kt[0] < itm.nt[1])
+                                    mma_block<D>(d + BN, qd + Q_SLOT, Q_HALF, k0, K_HALF, IDESC128);
+                            } else if (itm.nparts == 2) {
+                                mma_block<D>(d, k0, K_HALF, qd, Q_HALF, IDESC256);
+                            } else {
+                                mma_block<D>(d, k0, K_HALF, qd, Q_HALF, IDESC128);
+                            }
+                        } else if (pass == 0) {
+                            mma_block<D>(d, qd, Q_HALF, k0, K_HALF, IDESC128);
+                            if (nst == 2) mma_block<D>(d + BN, qd, Q_HALF, k1, K_HALF, IDESC128);
+                        } else if (mode == MODE_PACKED) {
+                            // head h's rows are Q rows 64h..64h+63 (64 rows = 8 KB = 512 units on)
+                            mma_block<D>(d, k0, K_HALF, qd, Q_HALF, IDESC64);
+                            if (nst == 2) mma_block<D>(d + BN + 64, k1, K_HALF, qd + 512, Q_HALF, IDESC64);
+                        } else {
+                            mma_block<D>(d, k0, K_HALF, qd, Q_HALF, IDESC128);
+                            if (nst == 2) mma_block<D>(d + BN, k1, K_HALF, qd, Q_HALF, IDESC128);
+                        }
+                        tc::mma_commit(&s.s_full[b]);
+                        tc::mma_commit(&s.empty[it % STAGES]);
+                        if (nst == 2) tc::mma_commit(&s.empty[(it + 1) % STAGES]);
                     }
-                    if (!wait_turn(&s.issued[gp], acc[gp], abort_flag) ||
-                        !tc::mbar_wait(&s.s_empty[gp][b], ((acc[gp] >> 1) & 1) ^ 1, abort_flag)) {
-                        ok = false;
-                        return;
-                    }
-                    tc::fence_after_sync();
-                    const uint32_t d_tmem = tmem + (uint32_t)((gp * 2 + b) * BN);
-                    const uint64_t qd = (itm.nr == 2 && gp == 1) ? qd1 : qd0;
-                    if (transposed)
-                        mma_kq<D, true>(d_tmem, qd, kd);
-                    else
-                        mma_kq<D, false>(d_tmem, qd, kd);
-                    tc::mma_commit(&s.s_full[gp][b]);
-                    ++acc[gp];
-                    *reinterpret_cast<volatile int*>(&s.issued[gp]) = acc[gp];
+                    it += nst;
+                    ++step;
                 }
-                if (issue) tc::mma_commit(&s.empty[stage]);
-                ++it;
-                ++local;
-            };
-            for (int kt = 0; ok && kt < itm.ntmax; ++kt) mma_tile(kt, false);
-            for (int kt = next_vis_tile(s.vis_before, 0, itm.ntmax); ok && kt < itm.ntmax;
-                 kt = next_vis_tile(s.vis_before, kt + 1, itm.ntmax))
-                mma_tile(kt, true);
-            // the item's Q tiles are free once these MMAs finish
-            tc::mma_commit(&s.q_empty[qb0]);
-            if (itm.nr == 2) tc::mma_commit(&s.q_empty[qb1]);
+            }
+            // the item's Q slots are free once both issuers' MMAs have finished
+            for (int r = 0; r < nslot; ++r) tc::mma_commit(&s.q_empty[mode == MODE_PAIR ? r : qs0]);
         }
         if (!ok) {
             s.abort_flag = 1;
@@ -549,15 +636,15 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
         tc::mbar_wait(&s.mma_done, 0, &s.never);
     }
 
-    // ------------------------------------------------------------ softmax groups
+    // ------------------------------------------------------------ softmax
     if (warp >= 2 && warp < MMA2_WARP) {
         const int sid = tid - 64;
         const int quarter = warp & 3;
-        const int grp = (warp - 2) >> 3;
-        const int wq = ((warp - 2) >> 2) & 1;               // which 64 columns of a tile
+        const int wi = (warp - 2) >> 2;                     // 0..3 within the lane quarter
         const int ln = quarter * 32 + lane;                 // this thread's TMEM lane
-        const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(wq * 64);
-        int acc_n = 0, u = 0;
+        const uint32_t tq = tmem + ((uint32_t)(quarter * 32) << 16);
+        const uint32_t lt_mask = (1u << lane) - 1u;
+        int step = 0;
         bool ok = true;
         for (int n = 0;; ++n) {
             // ---- the item, as fetched by the producer
@@ -575,89 +662,115 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
             tc::named_bar_sync(1, NSOFT);
             const int id = s.cur_item;
             if (id < 0) break;
-            const Item itm = item_info(p, s, id, npair, pair);
-            const int r = itm.nr == 2 ? grp : 0;          // this group's row tile
-            const int t = Item::pick(itm.t, r);
-            const int rows_t = Item::pick(itm.rows, r), rpg = Item::pick(itm.rpg, r);
-            const int n_mine = itm.nr == 2 ? Item::pick(itm.nt, r) : itm.ntmax;   // tiles with this group's rows
-            const int min_pos = Item::pick(itm.minp, r);
-            float* out = (T == 1) ? scores + (size_t)itm.lh * p.N_v
-                                  : score_part + ((size_t)itm.lh * T + t) * p.N_v;
+            const Item itm = item_info(p, s, mode, id);
 
-            // ---- rows of this group's row tile: lane 32q + i holds row q*rpg + i
-            if (wq == 0) {
-                const int rr = quarter * rpg + lane;
+            // ---- rows: lane 32q + i of row slot rs holds the part's row q*rpg + i
+            // (packed: lanes 64h + 32q' + i hold head h's row q'*rpg + i)
+            if (wi < (mode == MODE_PAIR ? itm.nparts : 1)) {
+                const int rs = wi;
+                int part, row;
+                if (mode == MODE_PACKED) {
+                    part = quarter >> 1;
+                    row = (quarter & 1) * itm.rpg[0] + lane;
+                } else {
+                    part = rs;
+                    row = quarter * Item::pick(itm.rpg, rs) + lane;
+                }
                 int pos = -1;
                 float wr = 0.f;
-                if (lane < rpg && rr < rows_t) {
-                    const int wi = (t * BM + rr) % p.n_win;
-                    pos = text_pos[wi];
+                const bool has = lane < Item::pick(itm.rpg, part) && row < Item::pick(itm.rows, part) &&
+                                 Item::pick(itm.lh, part) >= 0;
+                if (has) {
+                    const int t_row = mode == MODE_PAIR ? (2 * itm.pidx + rs) * BM : 0;
+                    const int wi_row = (t_row + row) % p.n_win;
+                    pos = text_pos[wi_row];
                     if (pos < 0 || pos >= p.N) pos = -1;
-                    wr = w[(long long)itm.l * p.w_stride + wi];
+                    wr = w[(long long)Item::pick(itm.l, part) * p.w_stride + wi_row];
                     if (!(wr >= 0.f) || isinf(wr)) {
                         raise_status(status, TGVKV_STATUS_WEIGHT);
                         wr = 0.f;
                     }
                 }
-                s.row_pos[grp][ln] = pos;
-                s.row_w[grp][ln] = wr;
+                s.row_pos[rs][ln] = pos;
+                s.row_w[rs][ln] = wr;
+            }
+            // the item's output rows start at zero: pass B adds two partial sums per key
+            for (int r = 0; r < itm.nparts; ++r) {
+                float* out = mode == MODE_PAIR
+                                 ? score_part + ((size_t)itm.lh[0] * p.T + 2 * itm.pidx + r) * p.N_v
+                                 : scores + (size_t)Item::pick(itm.lh, r) * p.N_v;
+                for (int vv = sid; vv < p.N_v; vv += NSOFT) out[vv] = 0.f;
             }
             tc::named_bar_sync(1, NSOFT);
-            const int my_pos = s.row_pos[grp][ln];
 
-            // ---- pass A: statistics of this thread's row over its 64 columns of its tiles
+            // ---- pass A: this warp's share of each step
+            // pair: row tile r = wi >> 1, columns 128r + 64(wi & 1) + [0, 64)
+            // single: K tile b = wi >> 1, columns 128b + 64(wi & 1) + [0, 64)
+            // packed: head b = quarter >> 1, columns 128b + 32 wi + [0, 32)
+            const int rsA = mode == MODE_PAIR ? (wi >> 1) : 0;
+            const int my_pos = s.row_pos[rsA][ln];
             float m = -INFINITY, z = 0.f, v = 0.f;
-            int local = 0;
-            for (int kt = 0; ok && kt < itm.ntmax; ++kt, ++local) {
-                const bool mine = itm.nr == 2 ? kt < n_mine : (local & 1) == grp;
-                if (!mine) continue;
-                const int b = acc_n & 1;
-                if (!warp_wait(&s.s_full[grp][b], (acc_n >> 1) & 1, abort_flag)) {
-                    ok = false;
-                    s.abort_flag = 1;
-                    break;
-                }
-                tc::fence_after_sync();
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    float x[32];
-                    tc::tmem_ld32(tl + (uint32_t)((grp * 2 + b) * BN + h * 32), x);
-                    tc::tmem_wait_ld();
-                    if (h == 1) {
-                        tc::fence_before_sync();
-                        __syncwarp();
-                        if (lane == 0) tc::mbar_arrive(&s.s_empty[grp][b]);
+            {
+                // Every warp runs every step of the item, also after a failed wait
+                // (then doing nothing), so that the warps of a quarter always meet
+                // at the same named barriers.
+                int cur = 0, kt[2];
+                while (next_step(itm, mode, 0, cur, s.vis_before, kt)) {
+                    const int b = step & 1;
+                    ++step;
+                    if (ok && !warp_wait(&s.s_full[b], ((step - 1) >> 1) & 1, abort_flag)) {
+                        ok = false;
+                        s.abort_flag = 1;
                     }
-                    const int lim = my_pos - (kt * BN + wq * 64 + h * 32);   // columns 0..lim visible
-                    if (lim >= 0) {
-                        const uint32_t vm = s.vmask[kt][wq * 2 + h];
-                        if (lim >= 31) {
-                            const float m_new = fmaxf(m, max32(x) * sl2);
-                            const float alpha = fast_exp2(m - m_new);
-                            z *= alpha;
-                            v *= alpha;
-                            exp_word<false>(x, sl2, -m_new, 31, vm, z, v);
-                            m = m_new;
-                        } else {
-                            const float m_new = fmaxf(m, max32_masked(x, lim) * sl2);
-                            const float alpha = fast_exp2(m - m_new);
-                            z *= alpha;
-                            v *= alpha;
-                            exp_word<true>(x, sl2, -m_new, lim, vm, z, v);
-                            m = m_new;
+                    if (!ok) continue;
+                    tc::fence_after_sync();
+                    int blk, ktile, cbase, nch;
+                    bool act;
+                    if (mode == MODE_PAIR) {
+                        blk = wi >> 1;
+                        ktile = kt[0];
+                        act = blk < itm.nparts && ktile < Item::pick(itm.nt, blk);
+                        cbase = 64 * (wi & 1);
+                        nch = 2;
+                    } else if (mode == MODE_SINGLE) {
+                        blk = wi >> 1;
+                        ktile = Item::pick(kt, blk);
+                        act = ktile >= 0;
+                        cbase = 64 * (wi & 1);
+                        nch = 2;
+                    } else {
+                        blk = quarter >> 1;
+                        ktile = Item::pick(kt, blk);
+                        act = ktile >= 0;
+                        cbase = 32 * wi;
+                        nch = 1;
+                    }
+                    if (!act) {
+                        release_acc(&s.s_empty[b], lane);
+                    } else {
+                        const uint32_t ta = tq + (uint32_t)(b * SCOLS + blk * BN + cbase);
+                        for (int ch = 0; ch < nch; ++ch) {
+                            float x[32];
+                            tc::tmem_ld32(ta + (uint32_t)(ch * 32), x);
+                            tc::tmem_wait_ld();
+                            if (ch == nch - 1) release_acc(&s.s_empty[b], lane);
+                            const int lim = my_pos - (ktile * BN + cbase + ch * 32);
+                            row_word(x, sl2, lim, s.vmask[ktile][(cbase >> 5) + ch], m, z, v);
                         }
                     }
                 }
-                ++acc_n;
             }
+
             // ---- combine the partial statistics of each row
-            s.part_m[grp * 2 + wq][ln] = m;
-            s.part_z[grp * 2 + wq][ln] = z;
-            s.part_v[grp * 2 + wq][ln] = v;
-            tc::named_bar_sync(1, NSOFT);
-            if (wq == 0) {
-                // one row tile: all four parts; two: this group's two
-                const int c0 = itm.nr == 2 ? grp * 2 : 0, c1 = itm.nr == 2 ? grp * 2 + 2 : 4;
+            s.part_m[wi][ln] = m;
+            s.part_z[wi][ln] = z;
+            s.part_v[wi][ln] = v;
+            tc::named_bar_sync(2 + quarter, 128);
+            // pair: warps 0 and 2 combine parts {0,1} / {2,3} of row slot 0 / 1;
+            // single and packed: warp 0 combines all four
+            if (mode == MODE_PAIR ? ((wi & 1) == 0 && (wi >> 1) < itm.nparts) : wi == 0) {
+                const int rs = mode == MODE_PAIR ? (wi >> 1) : 0;
+                const int c0 = mode == MODE_PAIR ? wi : 0, c1 = mode == MODE_PAIR ? wi + 2 : 4;
                 float mt = -INFINITY;
                 for (int c = c0; c < c1; ++c) mt = fmaxf(mt, s.part_m[c][ln]);
                 float zt = 0.f, vt = 0.f;
@@ -668,137 +781,151 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
                         vt += s.part_v[c][ln] * a;
                     }
                 }
-                const bool valid = my_pos >= 0 && zt > 0.f;
+                const bool valid = s.row_pos[rs][ln] >= 0 && zt > 0.f;
                 // rows without attention get -m' = -inf: every term 2^-inf = 0
-                s.row_nmp[grp][ln] =
-                    valid ? fast_log2(s.row_w[grp][ln] / ((float)p.G * zt)) - mt : -INFINITY;
-                s.row_mass[grp][ln] = valid ? vt / zt : 0.f;
+                s.row_nmp[rs][ln] =
+                    valid ? fast_log2(s.row_w[rs][ln] / ((float)p.G * zt)) - mt : -INFINITY;
+                s.row_mass[rs][ln] = valid ? vt / zt : 0.f;
             }
             tc::named_bar_sync(1, NSOFT);
-            if (wq == 0 && quarter == 0) {
-                // TV mass of this group's row tile, in lane order
-                float a = (s.row_mass[grp][lane] + s.row_mass[grp][lane + 32]) +
-                          (s.row_mass[grp][lane + 64] + s.row_mass[grp][lane + 96]);
+            if (sid < 64) {
+                // TV mass of each part, in lane order: pair -> row slot r over all
+                // lanes; packed -> head h over lanes 64h..64h+63; single -> all lanes
+                const int r = sid >> 5;
+                float a = 0.f;
+                if (mode == MODE_PAIR) {
+                    if (r < itm.nparts)
+                        a = (s.row_mass[r][lane] + s.row_mass[r][lane + 32]) +
+                            (s.row_mass[r][lane + 64] + s.row_mass[r][lane + 96]);
+                } else if (mode == MODE_PACKED) {
+                    a = s.row_mass[0][64 * r + lane] + s.row_mass[0][64 * r + 32 + lane];
+                } else if (r == 0) {
+                    a = (s.row_mass[0][lane] + s.row_mass[0][lane + 32]) +
+                        (s.row_mass[0][lane + 64] + s.row_mass[0][lane + 96]);
+                }
 #pragma unroll
                 for (int o = 16; o > 0; o >>= 1) a += __shfl_xor_sync(~0u, a, o);
-                if (lane == 0) s.tile_mass[grp] = a;
+                if (lane == 0) s.tile_mass[r] = a;
             }
 
-            // ---- pass B: text-weighted column sums, one key per thread
-            const float* nmp = s.row_nmp[grp] + wq * 64;
-            const int* rp = s.row_pos[grp] + wq * 64;
-            const bool full_groups = rpg == 32;
-            for (int kt = next_vis_tile(s.vis_before, 0, itm.ntmax); ok && kt < itm.ntmax;
-                 kt = next_vis_tile(s.vis_before, kt + 1, itm.ntmax), ++local) {
-                const bool mine = itm.nr == 2 ? kt < n_mine : (local & 1) == grp;
-                if (!mine) continue;
-                const int b = acc_n & 1;
-                if (!warp_wait(&s.s_full[grp][b], (acc_n >> 1) & 1, abort_flag)) {
-                    ok = false;
-                    s.abort_flag = 1;
-                    break;
-                }
-                tc::fence_after_sync();
-                const int j = kt * BN + ln;                     // this thread's key
-                const bool all_vis = kt * BN + BN - 1 <= min_pos;
-                float sum = 0.f;
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    float y[32];
-                    tc::tmem_ld32(tl + (uint32_t)((grp * 2 + b) * BN + h * 32), y);
-                    tc::tmem_wait_ld();
-                    if (h == 1) {
-                        tc::fence_before_sync();
-                        __syncwarp();
-                        if (lane == 0) tc::mbar_arrive(&s.s_empty[grp][b]);
-                    }
-                    if (full_groups)
-                        sum += colsum_group<true>(y, nmp + h * 32, rp + h * 32, sl2, rpg, j, all_vis);
-                    else
-                        sum += colsum_group<false>(y, nmp + h * 32, rp + h * 32, sl2, rpg, j, all_vis);
-                }
-                ++acc_n;
-                // the two column halves of key j meet at the wq == 0 warp of the group
-                const int b2 = u & 1;
-                const uint32_t ph = (u >> 1) & 1;
-                ++u;
-                if (wq == 1) {
-                    if (!warp_wait(&s.pb_empty[grp][quarter][b2], ph ^ 1, abort_flag)) {
+            // ---- pass B: text-weighted column sums, one key per lane
+            // pair: columns 64 wi + [0, 64) of the N = 256 product (row slot wi >> 1);
+            // single: K tile b = wi >> 1, columns 128b + 64(wi & 1) + [0, 64);
+            // packed: head b = wi >> 1, its rows' columns 128b + 64b + 32(wi & 1) + [0, 32).
+            // Each key gets exactly two partial sums (warps 2c and 2c+1), added
+            // atomically into an output row that starts at zero: 0 + a + b is the
+            // same in either order, so the result does not depend on timing.
+            // Pair items write one partial row per row tile.
+            {
+                int cur = 0, kt[2];
+                while (next_step(itm, mode, 1, cur, s.vis_before, kt)) {
+                    const int b = step & 1;
+                    if (ok && !warp_wait(&s.s_full[b], (step >> 1) & 1, abort_flag)) {
                         ok = false;
                         s.abort_flag = 1;
-                        break;
                     }
-                    s.pbuf[grp][b2][ln] = sum;
-                    __syncwarp();
-                    if (lane == 0) tc::mbar_arrive(&s.pb_full[grp][quarter][b2]);
-                } else {
-                    if (!warp_wait(&s.pb_full[grp][quarter][b2], ph, abort_flag)) {
-                        ok = false;
-                        s.abort_flag = 1;
-                        break;
+                    if (ok) tc::fence_after_sync();
+                    int blk, ktile, ccol, rcol, rs, nch, rpg, minp;
+                    bool act;
+                    if (mode == MODE_PAIR) {
+                        blk = 0;
+                        ktile = kt[0];
+                        rs = wi >> 1;
+                        act = rs < itm.nparts && ktile < Item::pick(itm.nt, rs);
+                        ccol = 64 * wi;
+                        rcol = 64 * (wi & 1);
+                        nch = 2;
+                        rpg = Item::pick(itm.rpg, rs);
+                        minp = Item::pick(itm.minp, rs);
+                    } else if (mode == MODE_SINGLE) {
+                        blk = wi >> 1;
+                        ktile = Item::pick(kt, blk);
+                        rs = 0;
+                        act = ktile >= 0;
+                        ccol = 128 * blk + 64 * (wi & 1);
+                        rcol = 64 * (wi & 1);
+                        nch = 2;
+                        rpg = itm.rpg[0];
+                        minp = itm.minp[0];
+                    } else {
+                        blk = wi >> 1;
+                        ktile = Item::pick(kt, blk);
+                        rs = 0;
+                        act = ktile >= 0;
+                        rcol = 64 * blk + 32 * (wi & 1);
+                        ccol = 128 * blk + rcol;
+                        nch = 1;
+                        rpg = itm.rpg[0];
+                        minp = itm.minp[0];
                     }
-                    sum += s.pbuf[grp][b2][ln];
-                    __syncwarp();
-                    if (lane == 0) tc::mbar_arrive(&s.pb_empty[grp][quarter][b2]);
-                    const uint32_t word = s.vmask[kt][quarter];
-                    if (j < p.N && ((word >> lane) & 1u)) {
-                        int vr = s.vis_before[kt] + __popc(word & ((1u << lane) - 1u));
-                        for (int q2 = 0; q2 < quarter; ++q2) vr += __popc(s.vmask[kt][q2]);
-                        if (vr < p.N_v) out[vr] = sum;
+                    float sum = 0.f;
+                    if (!ok) {
+                        // unwinding: no waits, no work, but the same barriers
+                    } else if (!act) {
+                        release_acc(&s.s_empty[b], lane);
+                    } else {
+                        const int j = ktile * BN + ln;               // this lane's key
+                        const bool all_vis = ktile * BN + BN - 1 <= minp;
+                        const uint32_t ta = tq + (uint32_t)(b * SCOLS + ccol);
+                        for (int ch = 0; ch < nch; ++ch) {
+                            float y[32];
+                            tc::tmem_ld32(ta + (uint32_t)(ch * 32), y);
+                            tc::tmem_wait_ld();
+                            if (ch == nch - 1) release_acc(&s.s_empty[b], lane);
+                            const float* nmp = s.row_nmp[rs] + rcol + ch * 32;
+                            const int* rp = s.row_pos[rs] + rcol + ch * 32;
+                            if (rpg >= 32)
+                                sum += colsum_group<true>(y, nmp, rp, sl2, rpg, j, all_vis);
+                            else
+                                sum += colsum_group<false>(y, nmp, rp, sl2, rpg, j, all_vis);
+                        }
                     }
+                    if (ok && act) {
+                        const uint32_t word = s.vmask[ktile][quarter];
+                        if ((word >> lane) & 1u) {
+                            const int vr = s.vq[ktile][quarter] + __popc(word & lt_mask);
+                            float* out = mode == MODE_PAIR
+                                             ? score_part + ((size_t)itm.lh[0] * p.T + 2 * itm.pidx + rs) * p.N_v
+                                             : scores + (size_t)Item::pick(itm.lh, mode == MODE_PACKED ? blk : 0) * p.N_v;
+                            if (vr < p.N_v) atomicAdd(out + vr, sum);
+                        }
+                    }
+                    ++step;
                 }
             }
-            // vision keys after every query row of this row tile get no attention
-            if (itm.nr == 2 || grp == 0)
-                for (int vv = s.vis_before[n_mine] + (sid & (GSOFT - 1)); vv < p.N_v; vv += GSOFT)
-                    out[vv] = 0.f;
-
-            // ---- reductions over row tiles (per head) and heads (per layer)
-            __threadfence();
+            // ---- per-head results; pairs of a head meet through a ticket
             if (sid == 0) s.stop = *abort_flag;
             tc::named_bar_sync(1, NSOFT);
             if (sid == 0) {
                 int last = 0;
-                if (T == 1) {
-                    stat_head[itm.lh] = s.tile_mass[0];
-                    last = 1;
+                if (mode != MODE_PAIR) {
+                    for (int h = 0; h < itm.nparts; ++h)
+                        stat_head[Item::pick(itm.lh, h)] = s.tile_mass[mode == MODE_PACKED ? h : 0];
                 } else {
-                    for (int rr = 0; rr < itm.nr; ++rr) {
-                        stat_part[(size_t)itm.lh * T + Item::pick(itm.t, rr)] =
-                            s.tile_mass[itm.nr == 2 ? rr : 0];
-                        __threadfence();
-                        if (atomicAdd(&tickets[itm.lh], 1u) == (unsigned)(T - 1)) last = 1;
-                    }
+                    for (int r = 0; r < itm.nparts; ++r)
+                        stat_part[(size_t)itm.lh[0] * p.T + 2 * itm.pidx + r] = s.tile_mass[r];
+                    // the barrier above ordered every thread's score writes before this fence
+                    __threadfence();
+                    const unsigned before = atomicAdd(&tickets[itm.lh[0]], (unsigned)itm.nparts);
+                    if (before + (unsigned)itm.nparts == (unsigned)p.T) last = 1;
                 }
                 s.head_last = last;
             }
             tc::named_bar_sync(1, NSOFT);
             if (s.head_last) {
+                // the last pair of a head adds the row tiles' partial rows in tile order
                 __threadfence();
-                if (T > 1) {
-                    for (int vv = sid; vv < p.N_v; vv += NSOFT) {
-                        float a = 0.f;
-                        for (int tt = 0; tt < T; ++tt)
-                            a += __ldcg(&score_part[((size_t)itm.lh * T + tt) * p.N_v + vv]);
-                        scores[(size_t)itm.lh * p.N_v + vv] = a;
-                    }
-                    if (sid == 0) {
-                        float a = 0.f;
-                        for (int tt = 0; tt < T; ++tt) a += __ldcg(&stat_part[(size_t)itm.lh * T + tt]);
-                        stat_head[itm.lh] = a;
-                        tickets[itm.lh] = 0u;
-                    }
+                const size_t base = (size_t)itm.lh[0] * p.T;
+                for (int vv = sid; vv < p.N_v; vv += NSOFT) {
+                    float a = 0.f;
+                    for (int t = 0; t < p.T; ++t) a += __ldcg(&score_part[(base + t) * p.N_v + vv]);
+                    scores[(size_t)itm.lh[0] * p.N_v + vv] = a;
                 }
                 if (sid == 0) {
-                    __threadfence();
-                    if (atomicAdd(&tickets[p.L * p.H_kv + itm.l], 1u) == (unsigned)(p.H_kv - 1)) {
-                        __threadfence();
-                        float S = 0.f;
-                        for (int gg = 0; gg < p.H_kv; ++gg)
-                            S += __ldcg(&stat_head[(size_t)itm.l * p.H_kv + gg]);
-                        tvb_stat[itm.l] = S;
-                        tickets[p.L * p.H_kv + itm.l] = 0u;
-                    }
+                    float a = 0.f;
+                    for (int t = 0; t < p.T; ++t) a += __ldcg(&stat_part[base + t]);
+                    stat_head[itm.lh[0]] = a;
+                    tickets[itm.lh[0]] = 0u;
                 }
             }
             const bool stop = s.stop;
@@ -814,6 +941,21 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
         __syncwarp();
         tc::fence_after_sync();
         tc::tmem_dealloc(tmem, TMEM_COLS);
+    }
+    // the last CTA to finish adds the per-head TV masses of each layer, in head order
+    if (tid == 0) {
+        __threadfence();
+        s.cta_last = atomicAdd(exit_counter, 1u) == gridDim.x - 1;
+    }
+    __syncthreads();
+    if (s.cta_last) {
+        __threadfence();
+        for (int l = tid; l < p.L; l += NTHREADS) {
+            float S = 0.f;
+            for (int g = 0; g < p.H_kv; ++g) S += __ldcg(&stat_head[(size_t)l * p.H_kv + g]);
+            tvb_stat[l] = S;
+        }
+        if (tid == 0) *exit_counter = 0u;
     }
 }
 
@@ -854,6 +996,30 @@ int sm_count() {
     return counts[dev];
 }
 
+template <int D, int MODE>
+cudaError_t launch_mode(const CUtensorMap& mq, const CUtensorMap& mk, const Problem& p, int n_items,
+                        const uint8_t* modality, const int32_t* text_pos, const float* w,
+                        float* scores, float* tvb_stat, char* ws, const WsLayout& lay,
+                        cudaStream_t stream) {
+    static_assert(sizeof(PSmem<D>) + 1024 <= 227 * 1024, "shared memory of one CTA");
+    const size_t smem = sizeof(PSmem<D>) + 1024;
+    cudaError_t e = cudaFuncSetAttribute(score_tc_kernel<D, MODE>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(score_tc_kernel<D, MODE>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                 (int)cudaSharedmemCarveoutMaxShared);
+    if (e != cudaSuccess) return e;
+    const int sms = sm_count();
+    if (sms <= 0) return cudaErrorInvalidDevice;
+    const int grid = n_items < sms ? n_items : sms;
+    score_tc_kernel<D, MODE><<<grid, NTHREADS, smem, stream>>>(
+        mq, mk, p, n_items, modality, text_pos, w, scores, tvb_stat,
+        reinterpret_cast<float*>(ws + lay.score_part), reinterpret_cast<float*>(ws + lay.stat_part),
+        reinterpret_cast<float*>(ws + lay.stat_head), reinterpret_cast<uint32_t*>(ws + lay.tickets),
+        reinterpret_cast<uint32_t*>(ws + lay.status));
+    return cudaGetLastError();
+}
+
 template <int D>
 cudaError_t launch_tc(const Problem& p, const uint16_t* q, const uint16_t* k,
                       const uint8_t* modality, const int32_t* text_pos, const float* w,
@@ -863,25 +1029,17 @@ cudaError_t launch_tc(const Problem& p, const uint16_t* q, const uint16_t* k,
     if (!make_map(&mq, q, (uint64_t)p.L * p.H_q * p.n_win, D, 32) ||
         !make_map(&mk, k, (uint64_t)p.L * p.H_kv * p.N, D, BN))
         return cudaErrorInvalidValue;
-    static_assert(sizeof(PSmem<D>) + 1024 <= 227 * 1024, "shared memory of one CTA");
-    const size_t smem = sizeof(PSmem<D>) + 1024;
-    cudaError_t e = cudaFuncSetAttribute(score_tc_kernel<D>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(score_tc_kernel<D>, cudaFuncAttributePreferredSharedMemoryCarveout,
-                                 (int)cudaSharedmemCarveoutMaxShared);
-    if (e != cudaSuccess) return e;
-    const int npair = p.T >= 2 ? (p.T + 1) / 2 : 1;
-    const int n_items = p.L * p.H_kv * npair;
-    const int sms = sm_count();
-    if (sms <= 0) return cudaErrorInvalidDevice;
-    const int grid = n_items < sms ? n_items : sms;
-    score_tc_kernel<D><<<grid, NTHREADS, smem, stream>>>(
-        mq, mk, p, modality, text_pos, w, scores, tvb_stat,
-        reinterpret_cast<float*>(ws + lay.score_part), reinterpret_cast<float*>(ws + lay.stat_part),
-        reinterpret_cast<float*>(ws + lay.stat_head), reinterpret_cast<uint32_t*>(ws + lay.tickets),
-        reinterpret_cast<uint32_t*>(ws + lay.status));
-    return cudaGetLastError();
+    // the item shape: pairs of row tiles, or one row tile per head, or two
+    // heads of at most 64 rows each packed into one row tile
+    const int LH = p.L * p.H_kv;
+    if (p.T >= 2)
+        return launch_mode<D, MODE_PAIR>(mq, mk, p, LH * score_pairs(p), modality, text_pos, w,
+                                         scores, tvb_stat, ws, lay, stream);
+    if (2 * p.R <= BM)
+        return launch_mode<D, MODE_PACKED>(mq, mk, p, (LH + 1) / 2, modality, text_pos, w, scores,
+                                           tvb_stat, ws, lay, stream);
+    return launch_mode<D, MODE_SINGLE>(mq, mk, p, LH, modality, text_pos, w, scores, tvb_stat, ws,
+                                       lay, stream);
 }
 
 }  // namespace
