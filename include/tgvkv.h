@@ -152,11 +152,11 @@ int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
 
 /* Number of CUDA kernels one tgvkv_evict call launches for this problem
  * (introspection for callers that budget launches, e.g. inside a captured
- * graph; the paper has no counterpart): normally 2 (score, then budget +
- * select + gather fused), 4 when the fused kernel's shared-memory table does
- * not fit (score, budget, select, compact), one fewer when the problem has no
- * query rows (the scores are then zero-filled with memsets).  Returns -1 on
- * bad arguments. */
+ * graph; the paper has no counterpart): normally 2 (scores with the layer
+ * budgets, then select + gather fused), 3 when the fused kernel's
+ * shared-memory table does not fit (select and compact separately).  A problem
+ * with no query rows zero-fills the scores with memsets and launches the
+ * budget kernel in place of the score kernel.  Returns -1 on bad arguments. */
 int tgvkv_evict_launches(const tgvkv_desc* desc);
 
 /* Zero `workspace` (asynchronously on `stream`).  Needed once after the

@@ -123,7 +123,7 @@ int do_score(const Problem& p, const uint16_t* q, const uint16_t* k, const uint8
              cudaStream_t st) {
     const WsLayout lay = layout_of(p);
     cudaError_t e = launch_score(p, q, k, modality, text_pos, w, scores, tvb_stat,
-                                 static_cast<char*>(ws), lay, st);
+                                 static_cast<char*>(ws), lay, -1, nullptr, st);
     return e == cudaSuccess ? TGVKV_OK : cuda_fail(e, "score launch");
 }
 
@@ -255,20 +255,25 @@ int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     const WsLayout lay = layout_of(p);
     uint32_t* status = status_of(workspace, lay);
+    // the score kernel's last CTA also derives the layer budgets
     cudaError_t e = launch_score(p, q_text, k, modality, text_pos, w, scores, tvb_stat,
-                                 static_cast<char*>(workspace), lay, st);
+                                 static_cast<char*>(workspace), lay, budget_total(p, ratio), budgets,
+                                 st);
     if (e != cudaSuccess) return cuda_fail(e, "score launch");
-    e = launch_budget_select_compact(p, scores, tvb_stat, budget_total(p, ratio), budgets,
-                                     modality, offsets, idx, k, v, k_out, v_out,
-                                     retained_rows(p, ratio), status, st);
-    if (e != cudaSuccess) return cuda_fail(e, "budget/select/compact launch");
+    if (score_launches(p) == 0) {   // no score kernel ran: split the (zero) statistic here
+        e = launch_budget(p, tvb_stat, budget_total(p, ratio), budgets, status, st);
+        if (e != cudaSuccess) return cuda_fail(e, "budget launch");
+    }
+    e = launch_select_compact(p, scores, budgets, modality, offsets, idx, k, v, k_out, v_out,
+                              retained_rows(p, ratio), status, st);
+    if (e != cudaSuccess) return cuda_fail(e, "select/compact launch");
     return ok();
 }
 
 int tgvkv_evict_launches(const tgvkv_desc* desc) {
     Problem p{};
     if (make_problem(desc, &p) != TGVKV_OK) return -1;
-    return score_launches(p) + budget_select_compact_launches(p);
+    return (score_launches(p) == 0 ? 1 : score_launches(p)) + select_compact_launches(p);
 }
 
 int tgvkv_workspace_init(const tgvkv_desc* desc, void* workspace, void* stream) {

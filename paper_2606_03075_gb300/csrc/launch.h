@@ -11,11 +11,13 @@
 namespace tgvkv {
 
 // TWR scores + TVB statistic (score_tc.cu).  The completion counters in the
-// workspace must be zero on entry; the kernel leaves them zero.
+// workspace must be zero on entry; the kernel leaves them zero.  When
+// `budgets` is not null, the CTA that finishes last also splits
+// `budget_total` over the layers (Eq. 5) into budgets[L].
 cudaError_t launch_score(const Problem& p, const uint16_t* q, const uint16_t* k,
                          const uint8_t* modality, const int32_t* text_pos, const float* w,
                          float* scores, float* tvb_stat, char* ws, const WsLayout& lay,
-                         cudaStream_t stream);
+                         long long budget_total, int32_t* budgets, cudaStream_t stream);
 
 cudaError_t launch_budget(const Problem& p, const float* tvb_stat, long long total,
                           int32_t* budgets, uint32_t* status, cudaStream_t stream);
@@ -24,21 +26,19 @@ cudaError_t launch_select(const Problem& p, const float* scores, const int32_t* 
                           const uint8_t* modality, int64_t* offsets, int32_t* idx,
                           uint32_t* status, cudaStream_t stream);
 
-// budget + select + gather fused (tgvkv_evict): one CTA per (layer, KV head)
-// derives all layer budgets from the TVB statistic, selects its set and
-// gathers its rows; falls back to the three separate kernels when the keys and
-// retained rows of a head do not fit in shared memory.
-cudaError_t launch_budget_select_compact(const Problem& p, const float* scores,
-                                         const float* tvb_stat, long long budget_total,
-                                         int32_t* budgets, const uint8_t* modality,
-                                         int64_t* offsets, int32_t* idx, const uint16_t* k,
-                                         const uint16_t* v, uint16_t* k_out, uint16_t* v_out,
-                                         long long capacity_rows, uint32_t* status,
-                                         cudaStream_t stream);
+// select + gather fused (tgvkv_evict): one CTA per (layer, KV head) selects
+// its set and gathers its rows; falls back to the separate select and compact
+// kernels when the keys and retained rows of a head do not fit in shared
+// memory.
+cudaError_t launch_select_compact(const Problem& p, const float* scores, const int32_t* budgets,
+                                  const uint8_t* modality, int64_t* offsets, int32_t* idx,
+                                  const uint16_t* k, const uint16_t* v, uint16_t* k_out,
+                                  uint16_t* v_out, long long capacity_rows, uint32_t* status,
+                                  cudaStream_t stream);
 
-// Kernels launch_score / launch_budget_select_compact launch for p.
+// Kernels launch_score / launch_select_compact launch for p.
 int score_launches(const Problem& p);
-int budget_select_compact_launches(const Problem& p);
+int select_compact_launches(const Problem& p);
 
 cudaError_t launch_compact(const Problem& p, const uint16_t* k, const uint16_t* v,
                            const int64_t* offsets, const int32_t* idx, uint16_t* k_out,

@@ -51,6 +51,7 @@
 
 #include <mutex>
 
+#include "budget.cuh"
 #include "common.cuh"
 #include "launch.h"
 #include "tc05.cuh"
@@ -346,7 +347,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
                 float* __restrict__ scores, float* __restrict__ tvb_stat,
                 float* __restrict__ score_part, float* __restrict__ stat_part,
                 float* __restrict__ stat_head, uint32_t* __restrict__ tickets,
-                uint32_t* __restrict__ status) {
+                uint32_t* __restrict__ status, long long budget_total, int32_t* __restrict__ budgets) {
     extern __shared__ unsigned char smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     PSmem<D>& s = *reinterpret_cast<PSmem<D>*>(smem_raw + (((raw + 1023u) & ~1023u) - raw));
@@ -462,7 +463,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
         tc::tma_prefetch_desc(&tmap_q);
         tc::tma_prefetch_desc(&tmap_k);
         int it = 0;
-        int qn[2] = {0, 0};
+        int qn0 = 0, qn1 = 0;     // uses of each Q slot
         bool ok = true;
         for (int n = 0; ok; ++n) {
             // fetch the next item (or the end mark) for every role of this CTA
@@ -489,11 +490,11 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
             const int nslot = mode == MODE_PAIR ? itm.nparts : 1;
             for (int r = 0; r < nslot; ++r) {
                 const int qs = mode == MODE_PAIR ? r : (n & 1);
-                if (!tc::mbar_wait(&s.q_empty[qs], (qn[qs] & 1) ^ 1, abort_flag)) {
+                const int use = qs ? qn1++ : qn0++;
+                if (!tc::mbar_wait(&s.q_empty[qs], (use & 1) ^ 1, abort_flag)) {
                     ok = false;
                     break;
                 }
-                ++qn[qs];
                 tc::mbar_arrive_expect_tx(&s.q_full[qs], 4 * (D / 64) * QBOX_BYTES);
 #pragma unroll
                 for (int qg = 0; qg < 4; ++qg) {
@@ -535,8 +536,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
             raise_status(status, TGVKV_STATUS_TIMEOUT);
         }
         // every copy this CTA issued has landed before it may exit
-        for (int qs = 0; qs < 2; ++qs)
-            if (qn[qs] > 0) tc::mbar_wait(&s.q_full[qs], (qn[qs] - 1) & 1, &s.never);
+        if (qn0 > 0) tc::mbar_wait(&s.q_full[0], (qn0 - 1) & 1, &s.never);
+        if (qn1 > 0) tc::mbar_wait(&s.q_full[1], (qn1 - 1) & 1, &s.never);
         for (int i = max(0, it - STAGES); i < it; ++i)
             tc::mbar_wait(&s.full[i % STAGES], (i / STAGES) & 1, &s.never);
     }
@@ -551,7 +552,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
         const uint64_t qdesc0 = tc::sdesc_k_sw128(smem_u32(&s.q[0][0][0]));
         constexpr uint32_t KSTAGE_DESC = (uint32_t)(sizeof(s.k[0]) >> 4);
         int it = 0, step = 0;
-        int qn[2] = {0, 0};
+        int qn0 = 0, qn1 = 0;     // uses of each Q slot
         bool ok = true;
         for (int n = 0; ok; ++n) {
             const int slot = n % NIQ;
@@ -567,11 +568,11 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
             const int qs0 = mode == MODE_PAIR ? 0 : (n & 1);
             for (int r = 0; r < nslot; ++r) {
                 const int qs = mode == MODE_PAIR ? r : qs0;
-                if (!tc::mbar_wait(&s.q_full[qs], qn[qs] & 1, abort_flag)) {
+                const int use = qs ? qn1++ : qn0++;
+                if (!tc::mbar_wait(&s.q_full[qs], use & 1, abort_flag)) {
                     ok = false;
                     break;
                 }
-                ++qn[qs];
             }
             if (!ok) break;
             const uint64_t qd = qdesc0 + (uint64_t)(qs0 * Q_SLOT);
@@ -955,6 +956,13 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
             for (int g = 0; g < p.H_kv; ++g) S += __ldcg(&stat_head[(size_t)l * p.H_kv + g]);
             tvb_stat[l] = S;
         }
+        if (budgets) {
+            // the layer budgets of Eq. 5, with the now idle K ring as scratch
+            __syncthreads();
+            static_assert(sizeof(BudgetScratch) <= sizeof(s.k), "budget scratch in the K ring");
+            tvb_budget_block(tvb_stat, p.L, budget_total, p.N_v, budgets, status,
+                             *reinterpret_cast<BudgetScratch*>(&s.k[0][0][0]));
+        }
         if (tid == 0) *exit_counter = 0u;
     }
 }
@@ -1000,7 +1008,7 @@ template <int D, int MODE>
 cudaError_t launch_mode(const CUtensorMap& mq, const CUtensorMap& mk, const Problem& p, int n_items,
                         const uint8_t* modality, const int32_t* text_pos, const float* w,
                         float* scores, float* tvb_stat, char* ws, const WsLayout& lay,
-                        cudaStream_t stream) {
+                        long long budget_total, int32_t* budgets, cudaStream_t stream) {
     static_assert(sizeof(PSmem<D>) + 1024 <= 227 * 1024, "shared memory of one CTA");
     const size_t smem = sizeof(PSmem<D>) + 1024;
     cudaError_t e = cudaFuncSetAttribute(score_tc_kernel<D, MODE>,
@@ -1016,7 +1024,7 @@ cudaError_t launch_mode(const CUtensorMap& mq, const CUtensorMap& mk, const Prob
         mq, mk, p, n_items, modality, text_pos, w, scores, tvb_stat,
         reinterpret_cast<float*>(ws + lay.score_part), reinterpret_cast<float*>(ws + lay.stat_part),
         reinterpret_cast<float*>(ws + lay.stat_head), reinterpret_cast<uint32_t*>(ws + lay.tickets),
-        reinterpret_cast<uint32_t*>(ws + lay.status));
+        reinterpret_cast<uint32_t*>(ws + lay.status), budget_total, budgets);
     return cudaGetLastError();
 }
 
@@ -1024,7 +1032,7 @@ template <int D>
 cudaError_t launch_tc(const Problem& p, const uint16_t* q, const uint16_t* k,
                       const uint8_t* modality, const int32_t* text_pos, const float* w,
                       float* scores, float* tvb_stat, char* ws, const WsLayout& lay,
-                      cudaStream_t stream) {
+                      long long budget_total, int32_t* budgets, cudaStream_t stream) {
     alignas(64) CUtensorMap mq, mk;
     if (!make_map(&mq, q, (uint64_t)p.L * p.H_q * p.n_win, D, 32) ||
         !make_map(&mk, k, (uint64_t)p.L * p.H_kv * p.N, D, BN))
@@ -1034,12 +1042,12 @@ cudaError_t launch_tc(const Problem& p, const uint16_t* q, const uint16_t* k,
     const int LH = p.L * p.H_kv;
     if (p.T >= 2)
         return launch_mode<D, MODE_PAIR>(mq, mk, p, LH * score_pairs(p), modality, text_pos, w,
-                                         scores, tvb_stat, ws, lay, stream);
+                                         scores, tvb_stat, ws, lay, budget_total, budgets, stream);
     if (2 * p.R <= BM)
         return launch_mode<D, MODE_PACKED>(mq, mk, p, (LH + 1) / 2, modality, text_pos, w, scores,
-                                           tvb_stat, ws, lay, stream);
+                                           tvb_stat, ws, lay, budget_total, budgets, stream);
     return launch_mode<D, MODE_SINGLE>(mq, mk, p, LH, modality, text_pos, w, scores, tvb_stat, ws,
-                                       lay, stream);
+                                       lay, budget_total, budgets, stream);
 }
 
 }  // namespace
@@ -1049,7 +1057,7 @@ int score_launches(const Problem& p) { return p.R == 0 ? 0 : 1; }
 cudaError_t launch_score(const Problem& p, const uint16_t* q, const uint16_t* k,
                          const uint8_t* modality, const int32_t* text_pos, const float* w,
                          float* scores, float* tvb_stat, char* ws, const WsLayout& lay,
-                         cudaStream_t stream) {
+                         long long budget_total, int32_t* budgets, cudaStream_t stream) {
     if (p.R == 0) {  // no query rows: no attention mass anywhere
         cudaError_t e = cudaSuccess;
         if (p.N_v > 0)
@@ -1058,8 +1066,10 @@ cudaError_t launch_score(const Problem& p, const uint16_t* q, const uint16_t* k,
         return e;
     }
     if (p.d == 64)
-        return launch_tc<64>(p, q, k, modality, text_pos, w, scores, tvb_stat, ws, lay, stream);
-    return launch_tc<128>(p, q, k, modality, text_pos, w, scores, tvb_stat, ws, lay, stream);
+        return launch_tc<64>(p, q, k, modality, text_pos, w, scores, tvb_stat, ws, lay, budget_total,
+                             budgets, stream);
+    return launch_tc<128>(p, q, k, modality, text_pos, w, scores, tvb_stat, ws, lay, budget_total,
+                          budgets, stream);
 }
 
 }  // namespace tgvkv

@@ -2,7 +2,8 @@
 // (layer, KV head) keeps every text position and the b_l vision positions of
 // highest score, ties to the lower position, in ascending position order --
 // and, in the fused form used by tgvkv_evict, gathers the retained K and V
-// rows straight away.
+// rows straight away.  The layer budgets come in from global memory (on the
+// evict path the score kernel derives them).
 //
 // Selection: the scores become order-preserving 32-bit keys in shared memory;
 // an MSB-first radix select (four 8-bit digits) finds the key T of the b_l-th
@@ -11,7 +12,6 @@
 // such keys in position order.  Each thread then owns a contiguous range of
 // positions; three block prefix sums (vision keys, keys equal to T, kept
 // positions) give every kept position its output slot.
-#include "budget.cuh"
 #include "common.cuh"
 #include "launch.h"
 
@@ -50,24 +50,26 @@ __device__ __forceinline__ int block_exclusive_scan(int x, int* buf, int* total)
     return res;
 }
 
-constexpr size_t kBudgetBytes = (sizeof(BudgetScratch) + 15) & ~size_t(15);
+// Shared memory of one CTA: keys [N_v], retained rows [N] (gather form) and
+// the modality bytes [N].
+__host__ __device__ inline size_t select_smem(const Problem& p, bool compact) {
+    return sizeof(uint32_t) * (size_t)p.N_v + (compact ? sizeof(int) * (size_t)p.N : 0) +
+           (((size_t)p.N + 15) & ~size_t(15));
+}
 
-// COMPACT: also gather the retained rows.  FUSED_BUDGET: derive the budgets
-// from the TVB statistic (every CTA runs the same deterministic split; CTA 0
-// writes them out) instead of reading them.
-template <bool COMPACT, bool FUSED_BUDGET, int VPR>
+// COMPACT: also gather the retained rows.
+template <bool COMPACT, int VPR>
 __global__ void __launch_bounds__(kThreads)
-tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __restrict__ budgets_in,
-                  const float* __restrict__ tvb_stat, long long budget_total,
-                  int32_t* __restrict__ budgets_out,
-                  const uint8_t* __restrict__ modality, int64_t* __restrict__ offsets,
+tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __restrict__ budgets,
+                  const uint8_t* __restrict__ modality_g, int64_t* __restrict__ offsets,
                   int32_t* __restrict__ idx, const uint4* __restrict__ k,
                   const uint4* __restrict__ v, uint4* __restrict__ k_out,
                   uint4* __restrict__ v_out, uint32_t* __restrict__ status) {
     extern __shared__ __align__(16) unsigned char dyn_raw[];
-    BudgetScratch& bs = *reinterpret_cast<BudgetScratch*>(dyn_raw);
-    uint32_t* keys = reinterpret_cast<uint32_t*>(dyn_raw + (FUSED_BUDGET ? kBudgetBytes : 0));  // [N_v]
+    uint32_t* keys = reinterpret_cast<uint32_t*>(dyn_raw);  // [N_v]
     int* rows = reinterpret_cast<int*>(keys + p.N_v);       // [N_t + b] (gather form)
+    uint8_t* modality = reinterpret_cast<uint8_t*>(dyn_raw) + sizeof(uint32_t) * (size_t)p.N_v +
+                        (COMPACT ? sizeof(int) * (size_t)p.N : 0);   // [N]
     __shared__ int hist[256];
     __shared__ int scan_buf[33];
     __shared__ uint32_t s_prefix;
@@ -77,12 +79,7 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
     const int lg = blockIdx.x, l = lg / p.H_kv, g = lg % p.H_kv;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 
-    const int32_t* budgets = budgets_in;
-    if (FUSED_BUDGET) {
-        tvb_budget_block(tvb_stat, p.L, budget_total, p.N_v, blockIdx.x == 0 ? budgets_out : nullptr,
-                         status, bs);
-        budgets = bs.result;
-    }
+    for (int j = tid; j < p.N; j += kThreads) modality[j] = __ldg(modality_g + j);
     int b = budgets[l];
     if (b < 0 || b > p.N_v) {
         if (tid == 0) raise_status(status, TGVKV_STATUS_BUDGET);
@@ -241,17 +238,17 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
     }
 }
 
-template <bool COMPACT, bool FUSED_BUDGET, int VPR>
-cudaError_t launch_sel(const Problem& p, const float* scores, const int32_t* budgets_in,
-                       const float* tvb_stat, long long budget_total, int32_t* budgets_out,
+template <bool COMPACT, int VPR>
+cudaError_t launch_sel(const Problem& p, const float* scores, const int32_t* budgets,
                        const uint8_t* modality, int64_t* offsets, int32_t* idx,
                        const uint16_t* k, const uint16_t* v, uint16_t* k_out, uint16_t* v_out,
-                       uint32_t* status, size_t smem, cudaStream_t stream) {
-    auto kern = tpr_select_kernel<COMPACT, FUSED_BUDGET, VPR>;
+                       uint32_t* status, cudaStream_t stream) {
+    auto kern = tpr_select_kernel<COMPACT, VPR>;
+    const size_t smem = select_smem(p, COMPACT);
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     kern<<<p.L * p.H_kv, kThreads, smem, stream>>>(
-        p, scores, budgets_in, tvb_stat, budget_total, budgets_out, modality, offsets, idx,
+        p, scores, budgets, modality, offsets, idx,
         reinterpret_cast<const uint4*>(k),
         reinterpret_cast<const uint4*>(v), reinterpret_cast<uint4*>(k_out),
         reinterpret_cast<uint4*>(v_out), status);
@@ -263,37 +260,29 @@ cudaError_t launch_sel(const Problem& p, const float* scores, const int32_t* bud
 cudaError_t launch_select(const Problem& p, const float* scores, const int32_t* budgets,
                           const uint8_t* modality, int64_t* offsets, int32_t* idx,
                           uint32_t* status, cudaStream_t stream) {
-    return launch_sel<false, false, 16>(p, scores, budgets, nullptr, -1, nullptr, modality, offsets,
-                                        idx, nullptr, nullptr, nullptr, nullptr, status,
-                                        sizeof(uint32_t) * (size_t)p.N_v, stream);
+    return launch_sel<false, 16>(p, scores, budgets, modality, offsets, idx, nullptr, nullptr, nullptr,
+                                 nullptr, status, stream);
 }
 
-int budget_select_compact_launches(const Problem& p) {
-    const size_t smem = kBudgetBytes + sizeof(uint32_t) * ((size_t)p.N_v + (size_t)p.N);
-    return smem > kFusedSmemLimit ? 3 : 1;
+int select_compact_launches(const Problem& p) {
+    return select_smem(p, true) > kFusedSmemLimit ? 2 : 1;
 }
 
-cudaError_t launch_budget_select_compact(const Problem& p, const float* scores,
-                                         const float* tvb_stat, long long budget_total,
-                                         int32_t* budgets, const uint8_t* modality,
-                                         int64_t* offsets, int32_t* idx, const uint16_t* k,
-                                         const uint16_t* v, uint16_t* k_out, uint16_t* v_out,
-                                         long long capacity_rows, uint32_t* status,
-                                         cudaStream_t stream) {
-    const size_t smem = kBudgetBytes + sizeof(uint32_t) * ((size_t)p.N_v + (size_t)p.N);
-    if (smem > kFusedSmemLimit) {
-        cudaError_t e = launch_budget(p, tvb_stat, budget_total, budgets, status, stream);
-        if (e == cudaSuccess)
-            e = launch_select(p, scores, budgets, modality, offsets, idx, status, stream);
+cudaError_t launch_select_compact(const Problem& p, const float* scores, const int32_t* budgets,
+                                  const uint8_t* modality, int64_t* offsets, int32_t* idx,
+                                  const uint16_t* k, const uint16_t* v, uint16_t* k_out,
+                                  uint16_t* v_out, long long capacity_rows, uint32_t* status,
+                                  cudaStream_t stream) {
+    if (select_smem(p, true) > kFusedSmemLimit) {
+        cudaError_t e = launch_select(p, scores, budgets, modality, offsets, idx, status, stream);
         if (e != cudaSuccess) return e;
         return launch_compact(p, k, v, offsets, idx, k_out, v_out, capacity_rows, status, stream);
     }
     if (p.d == 64)
-        return launch_sel<true, true, 8>(p, scores, nullptr, tvb_stat, budget_total, budgets,
-                                         modality, offsets, idx, k, v, k_out, v_out, status, smem,
-                                         stream);
-    return launch_sel<true, true, 16>(p, scores, nullptr, tvb_stat, budget_total, budgets, modality,
-                                      offsets, idx, k, v, k_out, v_out, status, smem, stream);
+        return launch_sel<true, 8>(p, scores, budgets, modality, offsets, idx, k, v, k_out, v_out,
+                                   status, stream);
+    return launch_sel<true, 16>(p, scores, budgets, modality, offsets, idx, k, v, k_out, v_out,
+                                status, stream);
 }
 
 }  // namespace tgvkv

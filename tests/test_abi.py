@@ -94,15 +94,16 @@ def test_host_budget_arithmetic_matches_oracle(lib):
 
 
 def test_evict_launch_count(lib):
-    """tgvkv_evict launches the score kernel and one fused budget/select/gather
-    kernel; four kernels only when the fused kernel's table (4 bytes per key)
-    would not fit shared memory; no score kernel without query rows."""
+    """tgvkv_evict launches the score kernel (which also derives the layer
+    budgets) and one fused select/gather kernel; select and compact run
+    separately when the fused kernel's tables would not fit shared memory;
+    without query rows the budget kernel replaces the score kernel."""
     ref = ctypes.byref
     for wl in synth.WORKLOADS.values():
         d = _desc(L=wl.L, H_q=wl.H_q, H_kv=wl.H_kv, d=wl.d, N=wl.N, N_v=wl.N_v, n_win=wl.n_win,
                   w_layer_stride=wl.n_win)
         assert lib.tgvkv_evict_launches(ref(d)) == 2, wl.name
-    assert lib.tgvkv_evict_launches(ref(_desc(N=32000, N_v=31000))) == 4
-    assert lib.tgvkv_evict_launches(ref(_desc(n_win=0))) == 1
+    assert lib.tgvkv_evict_launches(ref(_desc(N=32000, N_v=31000))) == 3
+    assert lib.tgvkv_evict_launches(ref(_desc(n_win=0))) == 2
     assert lib.tgvkv_evict_launches(ref(_desc(d=32))) == -1
     assert lib.tgvkv_evict_launches(None) == -1
