@@ -238,6 +238,203 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
     }
 }
 
+// ---- warp per (layer, KV head): select, emit and gather with warp-level
+// synchronisation only.  For shapes with many small heads: the warps of an SM
+// work on different heads and drift apart, so one warp's selection overlaps
+// other warps' gathers.  Shared memory per warp: keys [N_v], a 256-bin
+// histogram and the retained rows [N]; the modality bytes are shared by the CTA.
+__host__ __device__ inline size_t warp_select_words(const Problem& p) {
+    return (size_t)p.N_v + 256 + (size_t)p.N;
+}
+
+template <int VPR>
+__global__ void __launch_bounds__(256)
+tpr_select_warp_kernel(Problem p, const float* __restrict__ scores,
+                       const int32_t* __restrict__ budgets, const uint8_t* __restrict__ modality_g,
+                       int64_t* __restrict__ offsets, int32_t* __restrict__ idx,
+                       const uint4* __restrict__ k, const uint4* __restrict__ v,
+                       uint4* __restrict__ k_out, uint4* __restrict__ v_out,
+                       uint32_t* __restrict__ status) {
+    extern __shared__ __align__(16) unsigned char dyn_raw[];
+    const int wid = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nw = blockDim.x >> 5;
+    const size_t mod_bytes = ((size_t)p.N + 15) & ~size_t(15);
+    uint8_t* modality = dyn_raw;
+    uint32_t* keys = reinterpret_cast<uint32_t*>(dyn_raw + mod_bytes) + (size_t)wid * warp_select_words(p);
+    int* hist = reinterpret_cast<int*>(keys + p.N_v);
+    int* rows = hist + 256;
+    for (int j = threadIdx.x; j < p.N; j += blockDim.x) modality[j] = __ldg(modality_g + j);
+    __syncthreads();
+    const int lg = blockIdx.x * nw + wid;
+    if (lg >= p.L * p.H_kv) return;
+    const int l = lg / p.H_kv, g = lg % p.H_kv;
+    const uint32_t lt = (1u << lane) - 1u;
+
+    int b = budgets[l];
+    if (b < 0 || b > p.N_v) {
+        if (lane == 0) raise_status(status, TGVKV_STATUS_BUDGET);
+        b = b < 0 ? 0 : p.N_v;
+    }
+    const int len = p.N_t + b;
+    // CSR offset: rows of every (layer, head) before this one
+    long long off = 0;
+    for (int m = lane; m < l; m += 32) {
+        int bm = budgets[m];
+        bm = bm < 0 ? 0 : (bm > p.N_v ? p.N_v : bm);
+        off += (long long)p.H_kv * (p.N_t + bm);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) off += __shfl_xor_sync(~0u, off, o);
+    off += (long long)g * len;
+    if (lane == 0) {
+        offsets[lg] = off;
+        if (lg == p.L * p.H_kv - 1) offsets[lg + 1] = off + len;
+    }
+    const float* sc = scores + (size_t)lg * p.N_v;
+    for (int i = lane; i < p.N_v; i += 32) keys[i] = float_order_key(__ldg(sc + i));
+    __syncwarp();
+
+    // ---- radix select of the b-th largest key, 8 bits per round
+    uint32_t prefix = 0;
+    int kk = b;
+    if (b > 0) {
+        for (int shift = 24; shift >= 0; shift -= 8) {
+            for (int i = lane; i < 256; i += 32) hist[i] = 0;
+            __syncwarp();
+            const uint32_t hi_mask = (shift == 24) ? 0u : (0xFFFFFFFFu << (shift + 8));
+            for (int i = lane; i < p.N_v; i += 32) {
+                const uint32_t key = keys[i];
+                if ((key & hi_mask) == (prefix & hi_mask)) atomicAdd(&hist[(key >> shift) & 255], 1);
+            }
+            __syncwarp();
+            // lane t holds digits 255-8t .. 248-8t (highest first)
+            int cnt[8];
+            int sum = 0;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                cnt[e] = hist[255 - 8 * lane - e];
+                sum += cnt[e];
+            }
+            int incl = sum;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int y = __shfl_up_sync(~0u, incl, o);
+                if (lane >= o) incl += y;
+            }
+            const int above = incl - sum;
+            const bool here = above < kk && kk <= above + sum;
+            uint32_t digit = 0;
+            int rest = 0;
+            if (here) {
+                int a = above;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    if (kk <= a + cnt[e]) {
+                        digit = (uint32_t)(255 - 8 * lane - e);
+                        rest = kk - a;
+                        break;
+                    }
+                    a += cnt[e];
+                }
+            }
+            const int src = __ffs(__ballot_sync(~0u, here)) - 1;   // exactly one lane
+            digit = __shfl_sync(~0u, digit, src < 0 ? 0 : src);
+            rest = __shfl_sync(~0u, rest, src < 0 ? 0 : src);
+            prefix |= digit << shift;
+            kk = rest;
+            __syncwarp();
+        }
+    }
+    const bool none = (b == 0);
+    const uint32_t thr = prefix;
+    const int k_eq = none ? 0 : kk;
+
+    // ---- emission in position order, 32 positions per round
+    int vr_base = 0, eq_base = 0, out_base = 0;
+    for (int c0 = 0; c0 < p.N; c0 += 32) {
+        const int j = c0 + lane;
+        const bool in = j < p.N;
+        const bool isv = in && modality[j] != 0;
+        const uint32_t vb = __ballot_sync(~0u, isv);
+        const int vr = vr_base + __popc(vb & lt);
+        bool keep = in && !isv, eq = false;
+        if (isv && !none && vr < p.N_v) {
+            const uint32_t key = keys[vr];
+            if (key > thr) keep = true;
+            else if (key == thr) eq = true;
+        }
+        const uint32_t eb = __ballot_sync(~0u, eq);
+        if (eq && eq_base + __popc(eb & lt) < k_eq) keep = true;
+        const uint32_t kb = __ballot_sync(~0u, keep);
+        const int r = out_base + __popc(kb & lt);
+        if (keep && r < len) {
+            idx[off + r] = j;
+            rows[r] = j;
+        }
+        vr_base += __popc(vb);
+        eq_base += __popc(eb);
+        out_base += __popc(kb);
+    }
+    if (lane == 0 && out_base != len) raise_status(status, TGVKV_STATUS_COUNT);
+    __syncwarp();
+
+    // ---- gather the retained K and V rows
+    constexpr int RPI = 32 / VPR;   // rows per warp instruction
+    constexpr int UNROLL = 8;
+    const int n = min(len, out_base);
+    const int sub = lane / VPR, vec = lane % VPR;
+    const size_t head = (size_t)lg * p.N;
+    for (int r0 = 0; r0 < n; r0 += RPI * UNROLL) {
+        uint4 kr[UNROLL], vr[UNROLL];
+#pragma unroll
+        for (int u = 0; u < UNROLL; ++u) {
+            const int r = r0 + u * RPI + sub;
+            if (r < n) {
+                const size_t src = (head + rows[r]) * VPR + vec;
+                kr[u] = __ldg(k + src);
+                vr[u] = __ldg(v + src);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < UNROLL; ++u) {
+            const int r = r0 + u * RPI + sub;
+            if (r < n) {
+                const size_t dst = (size_t)(off + r) * VPR + vec;
+                k_out[dst] = kr[u];
+                v_out[dst] = vr[u];
+            }
+        }
+    }
+}
+
+// Warps per CTA of the warp-per-head kernel for p (0: use the CTA-per-head
+// kernel): only when there are many heads and eight heads' tables fit in
+// 64 KB, so that enough warps share an SM to keep the gather's loads in
+// flight (measured on GB300: faster for 1024 heads of 675 keys, slower for
+// 1024 heads of 3008 keys at four warps per CTA).
+inline int warp_select_warps(const Problem& p) {
+    const size_t per_warp = sizeof(uint32_t) * warp_select_words(p);
+    if (p.L * p.H_kv < 512) return 0;
+    return per_warp * 8 + (size_t)p.N <= 64 * 1024 ? 8 : 0;
+}
+
+template <int VPR>
+cudaError_t launch_sel_warp(const Problem& p, int nw, const float* scores, const int32_t* budgets,
+                            const uint8_t* modality, int64_t* offsets, int32_t* idx,
+                            const uint16_t* k, const uint16_t* v, uint16_t* k_out, uint16_t* v_out,
+                            uint32_t* status, cudaStream_t stream) {
+    auto kern = tpr_select_warp_kernel<VPR>;
+    const size_t smem = (((size_t)p.N + 15) & ~size_t(15)) + sizeof(uint32_t) * warp_select_words(p) * nw;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    const int heads = p.L * p.H_kv;
+    kern<<<(heads + nw - 1) / nw, nw * 32, smem, stream>>>(
+        p, scores, budgets, modality, offsets, idx, reinterpret_cast<const uint4*>(k),
+        reinterpret_cast<const uint4*>(v), reinterpret_cast<uint4*>(k_out),
+        reinterpret_cast<uint4*>(v_out), status);
+    return cudaGetLastError();
+}
+
 template <bool COMPACT, int VPR>
 cudaError_t launch_sel(const Problem& p, const float* scores, const int32_t* budgets,
                        const uint8_t* modality, int64_t* offsets, int32_t* idx,
@@ -265,7 +462,7 @@ cudaError_t launch_select(const Problem& p, const float* scores, const int32_t* 
 }
 
 int select_compact_launches(const Problem& p) {
-    return select_smem(p, true) > kFusedSmemLimit ? 2 : 1;
+    return warp_select_warps(p) == 0 && select_smem(p, true) > kFusedSmemLimit ? 2 : 1;
 }
 
 cudaError_t launch_select_compact(const Problem& p, const float* scores, const int32_t* budgets,
@@ -273,6 +470,13 @@ cudaError_t launch_select_compact(const Problem& p, const float* scores, const i
                                   const uint16_t* k, const uint16_t* v, uint16_t* k_out,
                                   uint16_t* v_out, long long capacity_rows, uint32_t* status,
                                   cudaStream_t stream) {
+    if (const int nw = warp_select_warps(p)) {
+        if (p.d == 64)
+            return launch_sel_warp<8>(p, nw, scores, budgets, modality, offsets, idx, k, v, k_out,
+                                      v_out, status, stream);
+        return launch_sel_warp<16>(p, nw, scores, budgets, modality, offsets, idx, k, v, k_out,
+                                   v_out, status, stream);
+    }
     if (select_smem(p, true) > kFusedSmemLimit) {
         cudaError_t e = launch_select(p, scores, budgets, modality, offsets, idx, status, stream);
         if (e != cudaSuccess) return e;

@@ -118,6 +118,30 @@ def test_queries_before_any_vision(api):
     assert g["budgets"].tolist() == oracle.tvb_budgets([0, 0, 0], 48, 64)
 
 
+# 512 (layer, KV head) pairs with 40 query rows each: packed score items (two
+# heads per row tile) and the warp-per-head select/gather of the evict path
+MANY = synth.custom("many_heads", 16, 32, 32, 64, [("text", 20), ("vision", 200), ("text", 40)],
+                    ratios=(0.3,))
+
+
+@pytest.mark.parametrize("ratio", [0.0, 0.3, 1.0])
+def test_many_small_heads(api, ratio):
+    g, _ = _full_check(api, MANY, ratio)
+    if ratio in (0.0, 1.0):
+        assert set(g["budgets"].tolist()) == ({0} if ratio == 0.0 else {MANY.N_v})
+
+
+def test_many_small_heads_all_ties(api):
+    """The warp-per-head selection when every vision score ties at zero: the
+    kept vision keys must be the lowest positions of each head."""
+    wl = synth.custom("many_early", 16, 32, 32, 64, [("text", 30), ("vision", 200), ("text", 10)],
+                      window=10, ratios=(0.25,))
+    inp = synth.generate(wl, seed=2)
+    inp["text_pos"] = np.arange(10, dtype=np.int32) * 3
+    g, _ = _full_check(api, wl, 0.25, inp=inp)
+    assert np.all(g["stat"] == 0) and np.all(g["scores"] == 0)
+
+
 def test_separate_calls_match_fused(api):
     wl = SMALL["ragged_gqa"]
     ratio = 0.1
