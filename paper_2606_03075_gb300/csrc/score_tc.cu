@@ -80,7 +80,9 @@ enum { MODE_PAIR = 0, MODE_SINGLE = 1, MODE_PACKED = 2 };
 template <int D>
 struct PSmem {
     uint16_t q[D / 64][2][BM * 64];          // two Q slots; per 64 dims, 128-byte-swizzled rows
-    uint16_t k[STAGES][D / 64][BN * 64];     // K ring
+    // K ring, stage-major within each 64 dims, so that the rows of stages 2j and
+    // 2j+1 are adjacent: single and packed steps multiply both in one N = 256 MMA
+    uint16_t k[D / 64][STAGES][BN * 64];
     uint64_t full[STAGES], empty[STAGES];
     uint64_t s_full[2], s_empty[2];
     uint64_t q_full[2], q_empty[2], mma_done;
@@ -353,7 +355,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
     PSmem<D>& s = *reinterpret_cast<PSmem<D>*>(smem_raw + (((raw + 1023u) & ~1023u) - raw));
     constexpr uint32_t KTILE_BYTES = (D / 64) * BN * 128;
     constexpr uint32_t QBOX_BYTES = 32 * 128;            // 32 rows x 64 dims
-    constexpr uint32_t K_HALF = BN * 64 * 2 / 16;        // 64-dim half of a K tile, 16-byte units
+    constexpr uint32_t K_HALF = STAGES * BN * 64 * 2 / 16;   // 64-dim half of the K ring, 16-byte units
     constexpr uint32_t Q_HALF = 2 * BM * 64 * 2 / 16;    // 64-dim half of the Q slots
     constexpr uint32_t Q_SLOT = BM * 64 * 2 / 16;
 
@@ -519,15 +521,28 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
                 tc::mbar_arrive_expect_tx(&s.full[stage], KTILE_BYTES);
 #pragma unroll
                 for (int h = 0; h < D / 64; ++h)
-                    tc::tma_load_2d(&s.k[stage][h][0], &tmap_k, h * 64, lh * p.N + kt * BN,
+                    tc::tma_load_2d(&s.k[h][stage][0], &tmap_k, h * 64, lh * p.N + kt * BN,
                                     &s.full[stage]);
+                ++it;
+            };
+            // a stage a step does not use (single / packed steps always take two)
+            auto skip = [&]() {
+                const int stage = it % STAGES;
+                if (!tc::mbar_wait(&s.empty[stage], ((it / STAGES) & 1) ^ 1, abort_flag)) {
+                    ok = false;
+                    return;
+                }
+                tc::mbar_arrive(&s.full[stage]);
                 ++it;
             };
             for (int pass = 0; ok && pass < 2; ++pass) {
                 int cur = 0, kt[2];
                 while (ok && next_step(itm, mode, pass, cur, s.vis_before, kt)) {
                     load(itm.lh[0], kt[0]);
-                    if (ok && kt[1] >= 0) load(mode == MODE_PACKED ? itm.lh[1] : itm.lh[0], kt[1]);
+                    if (ok && kt[1] >= 0)
+                        load(mode == MODE_PACKED ? itm.lh[1] : itm.lh[0], kt[1]);
+                    else if (ok && mode != MODE_PAIR)
+                        skip();
                 }
             }
         }
@@ -550,7 +565,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
         // (16-byte units, < 2^14 inside 256 KB) takes plain additions
         const uint64_t kdesc0 = tc::sdesc_k_sw128(smem_u32(&s.k[0][0][0]));
         const uint64_t qdesc0 = tc::sdesc_k_sw128(smem_u32(&s.q[0][0][0]));
-        constexpr uint32_t KSTAGE_DESC = (uint32_t)(sizeof(s.k[0]) >> 4);
+        constexpr uint32_t KSTAGE_DESC = BN * 64 * 2 / 16;   // one stage within a 64-dim half
         int it = 0, step = 0;
         int qn0 = 0, qn1 = 0;     // uses of each Q slot
         bool ok = true;
@@ -579,7 +594,10 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
             for (int pass = 0; ok && pass < 2; ++pass) {
                 int cur = 0, kt[2];
                 while (ok && next_step(itm, mode, pass, cur, s.vis_before, kt)) {
-                    const int nst = kt[1] >= 0 && mode != MODE_PAIR ? 2 : 1;
+                    // pair steps take one stage; single and packed steps two (an even
+                    // pair of adjacent stages), the second possibly unused
+                    const int nst = mode == MODE_PAIR ? 1 : 2;
+                    const bool has2 = kt[1] >= 0;
                     if ((step & 1) == me) {
                         const int b = step & 1;
                         bool got = tc::mbar_wait(&s.full[it % STAGES], (it / STAGES) & 1, abort_flag);
@@ -607,15 +625,15 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
                                 mma_block<D>(d, k0, K_HALF, qd, Q_HALF, IDESC128);
                             }
                         } else if (pass == 0) {
-                            mma_block<D>(d, qd, Q_HALF, k0, K_HALF, IDESC128);
-                            if (nst == 2) mma_block<D>(d + BN, qd, Q_HALF, k1, K_HALF, IDESC128);
+                            // Q against both adjacent K stages in one N = 256 product
+                            mma_block<D>(d, qd, Q_HALF, k0, K_HALF, has2 ? IDESC256 : IDESC128);
                         } else if (mode == MODE_PACKED) {
                             // head h's rows are Q rows 64h..64h+63 (64 rows = 8 KB = 512 units on)
                             mma_block<D>(d, k0, K_HALF, qd, Q_HALF, IDESC64);
-                            if (nst == 2) mma_block<D>(d + BN + 64, k1, K_HALF, qd + 512, Q_HALF, IDESC64);
+                            if (has2) mma_block<D>(d + BN + 64, k1, K_HALF, qd + 512, Q_HALF, IDESC64);
                         } else {
                             mma_block<D>(d, k0, K_HALF, qd, Q_HALF, IDESC128);
-                            if (nst == 2) mma_block<D>(d + BN, k1, K_HALF, qd, Q_HALF, IDESC128);
+                            if (has2) mma_block<D>(d + BN, k1, K_HALF, qd, Q_HALF, IDESC128);
                         }
                         tc::mma_commit(&s.s_full[b]);
                         tc::mma_commit(&s.empty[it % STAGES]);
