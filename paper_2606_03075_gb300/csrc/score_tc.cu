@@ -117,6 +117,17 @@ __device__ __forceinline__ int next_vis_tile(const int* vis_before, int kt, int 
     return kt;
 }
 
+// First global Q row of the 32-row box that lands in TMEM lanes 32g..32g+31
+// of Q slot r: pair / single -> part r's rows g*rpg..; packed -> head g/2's
+// rows (g%2)*rpg.. (an absent second head repeats the first's).
+__device__ __forceinline__ int q_box_row(const Item& it, int mode, int r, int g) {
+    if (mode == MODE_PACKED) {
+        const int h = (g >> 1) < it.nparts ? (g >> 1) : 0;
+        return Item::pick(it.qy, h) + (g & 1) * it.rpg[0];
+    }
+    return Item::pick(it.qy, r) + g * Item::pick(it.rpg, r);
+}
+
 template <int D>
 __device__ __forceinline__ Item item_info(const Problem& p, const PSmem<D>& s, int mode, int id) {
     Item it;
@@ -400,6 +411,9 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
         tc::tmem_relinquish();
     }
     const int n_tiles_all = (p.N + BN - 1) / BN;
+    // the first row positions are loaded now, so that their latency overlaps
+    // the modality loads below
+    const int pos0 = tid < p.R ? text_pos[tid % p.n_win] : -1;
     for (int kt = warp; kt < n_tiles_all; kt += NTHREADS / 32) {
         int cnt = 0;
 #pragma unroll
@@ -422,7 +436,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
     __syncthreads();
     tc::fence_after_sync();
     for (int r = tid; r < p.R; r += NTHREADS) {
-        const int pos = text_pos[r % p.n_win];
+        const int pos = r == tid ? pos0 : text_pos[r % p.n_win];
         if (pos >= 0 && pos < p.N) {
             atomicMax(&s.rt_max[r / BM], pos);
             atomicMin(&s.rt_min[r / BM], pos);
@@ -461,6 +475,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
     volatile int* abort_flag = &s.abort_flag;
 
     // ------------------------------------------------------------ producer
+    // Items are claimed from a counter in order, longest first (pair items
+    // differ in length); CTA c starts with item c without a claim.
     if (warp == 0 && lane == 0) {
         tc::tma_prefetch_desc(&tmap_q);
         tc::tma_prefetch_desc(&tmap_k);
@@ -474,7 +490,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
                 ok = false;
                 break;
             }
-            const int id = (int)atomicAdd(work_counter, 1u);
+            // the first item of CTA c is item c (grid <= items); later ones are claimed
+            const int id = n == 0 ? (int)blockIdx.x : (int)gridDim.x + (int)atomicAdd(work_counter, 1u);
             s.item_q[slot] = id < n_items ? id : -1;
             tc::mbar_arrive(&s.it_full[slot]);
             if (id >= n_items) {
@@ -500,13 +517,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
                 tc::mbar_arrive_expect_tx(&s.q_full[qs], 4 * (D / 64) * QBOX_BYTES);
 #pragma unroll
                 for (int qg = 0; qg < 4; ++qg) {
-                    int y;
-                    if (mode == MODE_PACKED) {
-                        const int h = (qg >> 1) < itm.nparts ? (qg >> 1) : 0;
-                        y = Item::pick(itm.qy, h) + (qg & 1) * itm.rpg[0];
-                    } else {
-                        y = Item::pick(itm.qy, r) + qg * Item::pick(itm.rpg, r);
-                    }
+                    const int y = q_box_row(itm, mode, r, qg);
 #pragma unroll
                     for (int h = 0; h < D / 64; ++h)
                         tc::tma_load_2d(&s.q[h][qs][qg * 32 * 64], &tmap_q, h * 64, y, &s.q_full[qs]);
