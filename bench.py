@@ -97,6 +97,20 @@ def stage_bytes(wl, ratio):
     }
 
 
+NOMINAL_HBM_GBS = 7900.0      # GB300 HBM3e, nominal
+NOMINAL_BF16_TFLOPS = 2250.0  # dense, nominal
+MUFU_EX2_PER_CLK_SM = 32      # ex2.approx.f32 results per clock per SM, measured on GB300
+GB300_SMS = 152
+
+
+def score_exps(wl):
+    """Exponentials of the score kernel's two passes: every (query row, visible
+    key) pair in pass A, every (query row, visible vision key) pair in pass B."""
+    pos = wl.text_pos.astype(np.int64)
+    vis_le = np.cumsum(wl.modality.astype(np.int64))[pos]
+    return int(wl.L * wl.H_q * ((pos + 1).sum() + vis_le.sum()))
+
+
 def score_flops(wl):
     """Algorithmic FLOPs of the score kernel: the logits q.k of every text-query
     row of every query head against each key it attends to (causal), once."""
@@ -255,24 +269,74 @@ def oracle_unit(wl, layer_inputs, l, g, ratio):
     oracle.compact(k[None, g:g + 1], v[None, g:g + 1], off, idx)
 
 
+_ONE_THREAD = {"OMP_NUM_THREADS": "1", "OPENBLAS_NUM_THREADS": "1", "MKL_NUM_THREADS": "1",
+               "BLIS_NUM_THREADS": "1", "VECLIB_MAXIMUM_THREADS": "1"}
+
+
+def _oracle_units_worker(job):
+    """Run the oracle on the given (layer, KV head) units and return the seconds
+    the oracle took (a process of its own, BLAS limited to one thread by the
+    environment; the inputs are drawn before the clock starts)."""
+    name, ratio, seed, units = job
+    wl = synth.WORKLOADS[name]
+    layers = {l: synth.draw_layer(wl, seed, l) for l in sorted({l for l, _ in units})}
+    t = time.perf_counter()
+    for l, g in units:
+        oracle_unit(wl, layers[l], l, g, ratio)
+    return time.perf_counter() - t
+
+
+def cpu_model():
+    try:
+        for line in open("/proc/cpuinfo"):
+            key = line.split(":")[0].strip().lower()
+            if key in ("model name", "cpu part", "hardware"):
+                return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    import platform
+    return platform.processor() or platform.machine()
+
+
 def run_cpu_baseline(wl, ratio, seed, seconds):
-    units, spent = 0, 0.0
-    for l in range(wl.L):
-        layer = synth.draw_layer(wl, seed, l)
-        for g in range(wl.H_kv):
-            t = time.perf_counter()
-            oracle_unit(wl, layer, l, g, ratio)
-            spent += time.perf_counter() - t
-            units += 1
-            if spent > seconds:
-                break
-        if spent > seconds:
-            break
-    us_per_layer = spent / units * wl.H_kv * 1e6
-    return {"value": us_per_layer, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
-            "sample": f"{units} (layer, KV head) units of {wl.name} in {spent:.1f} s "
-                      f"(fp64 numpy; BLAS may use all {os.cpu_count()} cores), scaled by "
-                      f"H_kv={wl.H_kv} per layer"}
+    """The fp64 oracle on this host: single-threaded, and on all cores (one
+    single-threaded process per core over (layer, KV head) units)."""
+    import multiprocessing as mp
+    cores = os.cpu_count() or 1
+    units = [(l, g) for l in range(wl.L) for g in range(wl.H_kv)]
+    saved = {k: os.environ.get(k) for k in _ONE_THREAD}
+    os.environ.update(_ONE_THREAD)
+    try:
+        ctx = mp.get_context("spawn")      # never fork after the GPU has been used
+        with ctx.Pool(1) as pool:          # single-threaded: grow the sample to ~seconds/2
+            n, spent1 = 1, 0.0
+            while True:
+                spent1 = pool.map(_oracle_units_worker, [(wl.name, ratio, seed, units[:n])])[0]
+                if spent1 > seconds / 2 or n >= len(units):
+                    break
+                n = min(len(units), max(n + 1, int(n * (seconds / 2) / max(spent1, 1e-3))))
+        single = spent1 / n * wl.H_kv * 1e6
+        # all cores: about seconds/4 of oracle work per process, all processes at once;
+        # the slowest process's time stands for the parallel wall time
+        per_core = max(1, int(n * 0.5))
+        jobs = [(wl.name, ratio, seed, [units[(c * per_core + i) % len(units)] for i in range(per_core)])
+                for c in range(cores)]
+        with ctx.Pool(cores) as pool:
+            pool.map(_oracle_units_worker, [(wl.name, ratio, seed, units[:1])] * cores, chunksize=1)
+            wall = max(pool.map(_oracle_units_worker, jobs, chunksize=1))
+        multi = wall / (cores * per_core) * wl.H_kv * 1e6
+    finally:
+        for k, v in saved.items():
+            if v is None:
+                os.environ.pop(k, None)
+            else:
+                os.environ[k] = v
+    return {"value": multi, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "single_thread_value": single, "cpu_model": cpu_model(),
+            "sample": f"fp64 numpy oracle, BLAS one thread per process: {n} (layer, KV head) "
+                      f"units of {wl.name} single-threaded ({spent1:.1f} s), then {per_core} "
+                      f"units on each of {cores} cores in parallel processes ({wall:.1f} s wall); "
+                      f"us/layer = time per unit x H_kv={wl.H_kv} (value: all cores)"}
 
 
 # --------------------------------------------------------------------------
@@ -489,6 +553,17 @@ def main():
                 "peak": hbm_peak, "unit": "GB/s",
                 "peak_source": f"{peak_src} hbm_gbs (MEASURED_PEAKS.json)"}
     roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["frac_nominal"] = roof["achieved"] / (NOMINAL_HBM_GBS if roof["bound"] == "hbm"
+                                               else NOMINAL_BF16_TFLOPS)
+    # the exponentials of the score kernel against the MUFU rate at the clock seen
+    clk_mhz = clocks.summary().get("sm_mhz") or float(peaks.get("sm_max_mhz", 2070.0))
+    exps = score_exps(wl)
+    mufu = {"exps_per_launch": exps,
+            "achieved_G_per_s": exps / (stage_ms["score"] * 1e-3) / 1e9,
+            "peak_G_per_s": MUFU_EX2_PER_CLK_SM * GB300_SMS * clk_mhz * 1e6 / 1e9,
+            "peak_source": f"{MUFU_EX2_PER_CLK_SM} ex2/clk/SM measured x {GB300_SMS} SMs x "
+                           f"{clk_mhz:.0f} MHz median under load"}
+    mufu["frac"] = mufu["achieved_G_per_s"] / mufu["peak_G_per_s"]
     sbytes, rows = step_bytes(wl, ratio)
     step_gbs = sbytes * args.steps * world / (region_ms * 1e-3) / 1e9
 
@@ -509,12 +584,14 @@ def main():
                            parallelism=f"replicas x{world}"),
             "hbm_step": {"bytes_per_step": sbytes, "bytes_per_layer": sbytes / wl.L,
                          "gbs": step_gbs, "peak": hbm_peak, "frac": step_gbs / hbm_peak,
+                         "frac_nominal": step_gbs / NOMINAL_HBM_GBS,
                          "definition": "K read once + compacted K/V written, per step"},
             "roofline": {"bound": roof["bound"], "kernel": dom, "achieved": roof["achieved"],
                          "peak": roof["peak"], "unit": roof["unit"], "frac": roof["frac"],
                          "traffic": traffic, "bytes_per_launch": sb[dom],
                          "flops_per_launch": flops, "launch_ms": stage_ms[dom],
-                         "peak_source": roof["peak_source"]},
+                         "peak_source": roof["peak_source"], "frac_nominal": roof["frac_nominal"]},
+            "score_mufu": mufu,
             "stage_ms": stage_ms,
             "fused_tail_ms": statistics.mean(step_ms) - stage_ms["score"],
             "step_ms_median": statistics.median(step_ms),

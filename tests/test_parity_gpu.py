@@ -293,3 +293,44 @@ def test_full_size_sampled(api, name, ratio, layers):
     P.check_selection_and_compaction(wl, inp, g, layers, ref_scores=ref_s)
     assert g["offsets"][-1] == wl.H_kv * (wl.L * wl.N_t + total)
     assert np.all(np.diff(g["offsets"]) == np.repeat(wl.N_t + g["budgets"], wl.H_kv))
+
+
+def test_layer_sharded_ranks_match_full_evict(api):
+    """The host logic of layer sharding with the CUDA backend: two ranks'
+    layer ranges scored separately, their statistics concatenated in rank
+    order (what the all-gather returns), budgets from the full vector, each
+    range selected and gathered on its own -- bit-identical to one full
+    tgvkv_evict.  The ranks run one after another here; nothing waits on
+    another rank's kernel."""
+    from paper_2606_03075_gb300 import shard
+    wl = synth.custom("shard_gqa", 5, 8, 2, 128,
+                      [("text", 11), ("vision", 300), ("text", 9), ("vision", 140),
+                       ("text", 33)], weights="dirichlet", ratios=(0.15,))
+    inp = synth.generate(wl, seed=3)
+    dev = P.device_inputs(inp)
+    full = P.run_evict(api, wl, inp, 0.15, dev)
+    assert full["status"] == 0
+    desc_full = api.desc_for_workload(wl)
+    backend = shard.CudaBackend("cuda")
+    world, stats, scores, spans = 2, [], [], []
+    for r in range(world):
+        l0, l1 = shard.layer_range(wl.L, r, world)
+        d = api.make_desc(l1 - l0, wl.H_q, wl.H_kv, wl.d, wl.N, wl.N_v, wl.n_win, 0.0, wl.n_win)
+        s, st = backend.score(d, dev["q"][l0:l1].contiguous(), dev["k"][l0:l1].contiguous(),
+                              dev["modality"], dev["text_pos"], dev["w"][l0:l1].contiguous())
+        stats.append(st), scores.append(s), spans.append((l0, l1, d))
+    full_stat = torch.cat(stats)
+    np.testing.assert_array_equal(full_stat.cpu().numpy(), full["stat"])
+    budgets = backend.budget(desc_full, full_stat, 0.15)
+    np.testing.assert_array_equal(budgets.cpu().numpy(), full["budgets"])
+    H = wl.H_kv
+    for (l0, l1, d), s in zip(spans, scores):
+        np.testing.assert_array_equal(s.cpu().numpy(), full["scores"][l0:l1])
+        off, idx, ko, vo = backend.select_compact(d, s, budgets[l0:l1].contiguous(), dev["modality"],
+                                                  dev["k"][l0:l1].contiguous(),
+                                                  dev["v"][l0:l1].contiguous())
+        lo, hi = full["offsets"][l0 * H], full["offsets"][l1 * H]
+        np.testing.assert_array_equal(off.cpu().numpy(), full["offsets"][l0 * H:l1 * H + 1] - lo)
+        np.testing.assert_array_equal(idx.cpu().numpy(), full["idx"][lo:hi])
+        np.testing.assert_array_equal(ko.view(torch.int16).cpu().numpy(), full["k_out"][lo:hi])
+        np.testing.assert_array_equal(vo.view(torch.int16).cpu().numpy(), full["v_out"][lo:hi])
