@@ -28,6 +28,26 @@ What is computed, in the paper's order (Section 3.3, "TGV-KV"):
    score (ties to the lower position), in ascending position order.
 7. Compaction: the K and V rows of the retained positions, copied bit for bit.
 
+Beyond that hot path (same file, same conventions):
+
+8. Text scores (Eq. 9): ``s^T_{l,t} = sum_{i} A_{i,t}`` over the query rows
+   for every text key t (rows before t contribute 0 through the causal mask),
+   per KV head as the mean over its G query heads, like Eq. 8.
+9. Derived text weights (Eq. 7): for the query row j (itself a text token at
+   position p_j), ``w_{l,j} = sum_{i >= j} A_{i,p_j} / (n_win - j)`` -- the
+   column sum of the text-text slice over the rows at or after j, divided by
+   their number -- averaged over the H_q query heads of the layer and then
+   L1-normalised over j to give w~ (the paper leaves the normalisation
+   unstated; the sum is the reading taken here).
+10. All-token budget basis: ``B = floor(r * N * L + 1/2)`` rows per head over
+   all layers, split by the same Eq. 5 rule with cap N.
+11. TPR with both cases of Eq. 10 and sink tokens: if b_l > N_t every text
+   position is kept plus the top (b_l - N_t) vision positions by s^V;
+   otherwise the top b_l text positions by s^T and no vision.  Sink positions
+   (the first ``keep_first`` and last ``keep_last`` tokens, Appendix A.2
+   "Implementation Details") are always kept and count against the part of the
+   budget of their own modality.
+
 Floating point: inputs are bf16 bit patterns widened exactly to float64; all
 arithmetic is float64.  The paper states no precision.
 
@@ -108,11 +128,56 @@ def twr_scores_tvb_stat(q: np.ndarray, k: np.ndarray, modality: np.ndarray,
 
 
 # --------------------------------------------------------------------------
+# Eq. 9 text scores and Eq. 7 derived text weights
+# --------------------------------------------------------------------------
+def text_scores_and_weights(q: np.ndarray, k: np.ndarray, modality: np.ndarray,
+                            text_pos: np.ndarray, scale: float, n_kv_heads: int,
+                            layers=None):
+    """Text-key importance (Eq. 9) and the normalised text weights (Eq. 7).
+
+    q, k, modality, text_pos as in twr_scores_tvb_stat; every query row must
+    sit on a text token.  Returns (text_scores [L, H_kv, N_t], weights
+    [L, n_win]):
+      text_scores[l, g, t] = (1/G) sum_{h in g} sum_i A_{l,h}[i, t]        (Eq. 9)
+      w_{l,j} = (1/H_q) sum_h sum_{i >= j} A_{l,h}[i, p_j] / (n_win - j)   (Eq. 7)
+      weights[l, j] = w_{l,j} / sum_j' w_{l,j'}
+    where t runs over the text keys in position order.
+    """
+    modality = np.asarray(modality)
+    text_pos = np.asarray(text_pos)
+    if np.any(modality[text_pos] != 0):
+        raise ValueError("a query row sits on a vision token")
+    n_layers, n_q_heads, n_win = q.shape[0], q.shape[1], q.shape[2]
+    group = n_q_heads // n_kv_heads
+    text = np.flatnonzero(modality == 0)
+    t_scores = np.zeros((n_layers, n_kv_heads, text.size))
+    weights = np.zeros((n_layers, n_win))
+    rows_at_or_after = n_win - np.arange(n_win)          # |{i : i >= j}|
+    for l in (range(n_layers) if layers is None else layers):
+        w_sum = np.zeros(n_win)
+        for h in range(n_q_heads):
+            g = h // group
+            a = causal_text_attention(q[l, h], k[l, g], text_pos, scale)
+            a_tt = a[:, text]                            # the text-text slice of A_l
+            t_scores[l, g] += a_tt.sum(axis=0) / group   # Eq. 9, mean over the group
+            w_sum += a[:, text_pos].sum(axis=0)          # Eq. 7 numerators (rows i >= j)
+        w = w_sum / n_q_heads / rows_at_or_after
+        weights[l] = w / w.sum()
+    return t_scores, weights
+
+
+# --------------------------------------------------------------------------
 # TVB: per-layer budgets from the statistic (Eq. 5)
 # --------------------------------------------------------------------------
 def vision_budget_total(ratio: float, n_vision: int, n_layers: int) -> int:
     """B_V = floor(r * N_v * L + 1/2): vision KV kept over all layers."""
     return int(math.floor(ratio * float(n_vision * n_layers) + 0.5))
+
+
+def all_budget_total(ratio: float, n_tokens: int, n_layers: int) -> int:
+    """B = floor(r * N * L + 1/2): KV rows kept per head over all layers when the
+    ratio counts every token (the main-text setting of Table 4)."""
+    return int(math.floor(ratio * float(n_tokens * n_layers) + 0.5))
 
 
 def tvb_budgets(stat, total: int, cap: int) -> list[int]:
@@ -188,6 +253,58 @@ def tpr_select(scores: np.ndarray, budgets, modality: np.ndarray):
     return np.asarray(offsets, dtype=np.int64), idx
 
 
+def sink_positions(n_tokens: int, keep_first: int, keep_last: int) -> np.ndarray:
+    """The always-kept positions: the first keep_first and the last keep_last."""
+    first = np.arange(min(keep_first, n_tokens))
+    last = np.arange(max(0, n_tokens - keep_last), n_tokens)
+    return np.union1d(first, last).astype(np.int64)
+
+
+def tpr_select_general(v_scores: np.ndarray, t_scores, budgets, modality: np.ndarray,
+                       keep_first: int = 0, keep_last: int = 0, vision_basis: bool = False):
+    """Retained positions per (layer, KV head) by both cases of Eq. 10, with sinks.
+
+    v_scores: [L, H_kv, N_v] vision scores s^V; t_scores: [L, H_kv, N_t] text
+    scores s^T (only read for layers with b_l <= N_t).  budgets: [L] rows b_l
+    of each head of layer l over all tokens.
+      b_l > N_t:  every text position, plus the (b_l - N_t) top vision positions
+      b_l <= N_t: the b_l top text positions, no vision position
+    With vision_basis the budgets count vision rows only and the first case
+    holds for every layer (b_l vision slots on top of all text; t_scores is not
+    read).  Ranking is (score descending, position ascending).  Sinks are kept
+    in any case; a sink of the ranked modality takes one of its slots (if slots
+    are fewer than sinks, every sink is still kept).  Returns CSR (offsets,
+    idx), positions ascending within a head.
+    """
+    modality = np.asarray(modality)
+    vision = np.flatnonzero(modality == 1)
+    text = np.flatnonzero(modality == 0)
+    n_tokens = modality.size
+    sinks = sink_positions(n_tokens, keep_first, keep_last)
+    is_sink = np.zeros(n_tokens, bool)
+    is_sink[sinks] = True
+    n_layers, n_kv_heads = v_scores.shape[0], v_scores.shape[1]
+    offsets = [0]
+    kept = []
+    for l in range(n_layers):
+        b = int(budgets[l])
+        for g in range(n_kv_heads):
+            if vision_basis or b > text.size:
+                slots = b if vision_basis else b - text.size
+                cand, s, always = vision, v_scores[l, g], text
+            else:
+                cand, s, slots, always = text, t_scores[l, g], b, np.zeros(0, np.int64)
+            free = ~is_sink[cand]
+            slots = max(0, slots - int(np.count_nonzero(~free)))
+            order = np.lexsort((cand[free], -s[free]))          # score desc, pos asc
+            chosen = cand[free][order[:slots]]
+            rows = np.union1d(np.union1d(always, sinks), chosen)
+            kept.append(rows.astype(np.int64))
+            offsets.append(offsets[-1] + rows.size)
+    idx = np.concatenate(kept) if kept else np.zeros(0, np.int64)
+    return np.asarray(offsets, dtype=np.int64), idx
+
+
 # --------------------------------------------------------------------------
 # Compaction of the retained KV
 # --------------------------------------------------------------------------
@@ -219,20 +336,47 @@ def compacted_kv_bytes(offsets, head_dim: int, elem_bytes: int = 2) -> int:
 # the whole step
 # --------------------------------------------------------------------------
 def evict(q_bits, k_bits, v_bits, modality, text_pos, w, ratio: float,
-          n_kv_heads: int, scale: float | None = None):
-    """Score, budget, select and compact, all in float64 on the host."""
+          n_kv_heads: int, scale: float | None = None, weights: str = "given",
+          basis: str = "vision", keep_first: int = 0, keep_last: int = 0):
+    """Score, budget, select and compact, all in float64 on the host.
+
+    weights: "given" uses ``w``; "eq7" derives w~ by Eq. 7 (``w`` is ignored).
+    basis:   "vision" -- r counts vision KV and every text KV is kept (case
+             b_l > N_t of Eq. 10 throughout); "all" -- r counts every KV and
+             Eq. 10 applies per layer with the text scores of Eq. 9.
+    """
     q = widen_bf16(q_bits)
     k = widen_bf16(k_bits)
     d = q.shape[-1]
     if scale is None:
         scale = 1.0 / math.sqrt(d)
+    modality = np.asarray(modality)
+    n_layers = q.shape[0]
+    n_tokens = modality.size
+    n_vision = int(np.count_nonzero(modality == 1))
+    t_scores = None
+    if weights == "eq7" or basis == "all":
+        t_scores, w_eq7 = text_scores_and_weights(q, k, modality, text_pos, scale, n_kv_heads)
+        if weights == "eq7":
+            w = w_eq7
     w = np.asarray(w, dtype=np.float64)
     scores, stat = twr_scores_tvb_stat(q, k, modality, text_pos, w, scale, n_kv_heads)
-    n_layers = q.shape[0]
-    n_vision = int(np.count_nonzero(np.asarray(modality) == 1))
-    total = vision_budget_total(ratio, n_vision, n_layers)
-    budgets = tvb_budgets(stat, total, n_vision)
-    offsets, idx = tpr_select(scores, budgets, modality)
+    if basis == "vision":
+        total = vision_budget_total(ratio, n_vision, n_layers)
+        budgets = tvb_budgets(stat, total, n_vision)
+        if keep_first or keep_last:
+            offsets, idx = tpr_select_general(scores, None, budgets, modality, keep_first,
+                                              keep_last, vision_basis=True)
+        else:
+            offsets, idx = tpr_select(scores, budgets, modality)
+    else:
+        total = all_budget_total(ratio, n_tokens, n_layers)
+        budgets = tvb_budgets(stat, total, n_tokens)
+        offsets, idx = tpr_select_general(scores, t_scores, budgets, modality, keep_first,
+                                          keep_last)
     k_out, v_out = compact(k_bits, v_bits, offsets, idx)
-    return dict(scores=scores, stat=stat, budgets=np.asarray(budgets, np.int64),
-                offsets=offsets, idx=idx, k_out=k_out, v_out=v_out)
+    out = dict(scores=scores, stat=stat, budgets=np.asarray(budgets, np.int64),
+               offsets=offsets, idx=idx, k_out=k_out, v_out=v_out, w=w)
+    if t_scores is not None:
+        out["text_scores"] = t_scores
+    return out

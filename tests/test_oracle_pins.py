@@ -370,3 +370,208 @@ def test_rows_normalised_independently_wide_range():
     assert np.allclose(a.sum(axis=1), 1.0, rtol=0, atol=1e-12)
     assert a[0, 3] > 1.0 - 1e-12
     assert np.all(np.abs(a[1] - 1.0 / 6.0) < 0.01)
+
+
+# ---------------------------------------------------------------- Eq. 7 / Eq. 9
+def _scalar_attention_rows(q, k, pos, scale, l, h, g):
+    """A_{l,h}[i, j] for j <= pos[i], by scalar loops (math.exp)."""
+    rows = []
+    for i, p in enumerate(pos):
+        logits = []
+        for j in range(p + 1):
+            dot = 0.0
+            for c in range(q.shape[-1]):
+                dot += q[l, h, i, c] * k[l, g, j, c]
+            logits.append(scale * dot)
+        mx = max(logits)
+        e = [math.exp(x - mx) for x in logits]
+        z = sum(e)
+        rows.append([x / z for x in e])
+    return rows
+
+
+def test_text_scores_and_weights_brute_force_tiny():
+    """Eq. 9 and Eq. 7 summed term by term over scalar attention entries."""
+    L, H_q, H_kv, d = 2, 4, 2, 5
+    q, k, modality, pos, _ = _rand_case(L, H_q, H_kv, d, seed=31)
+    scale = 0.53
+    ts, wt = oracle.text_scores_and_weights(q, k, modality, pos, scale, H_kv)
+    G = H_q // H_kv
+    trank = {}
+    for j, m in enumerate(modality):
+        if m == 0:
+            trank[j] = len(trank)
+    n_win = len(pos)
+    bts = np.zeros_like(ts)
+    bw = np.zeros((L, n_win))
+    for l in range(L):
+        num = [0.0] * n_win
+        for h in range(H_q):
+            g = h // G
+            a = _scalar_attention_rows(q, k, pos, scale, l, h, g)
+            for i, p in enumerate(pos):
+                for j in range(p + 1):
+                    if modality[j] == 0:
+                        bts[l, g, trank[j]] += a[i][j] / G
+                for jr in range(n_win):              # Eq. 7: rows i >= jr, column pos[jr]
+                    if i >= jr:
+                        num[jr] += a[i][pos[jr]]
+        raw = [num[jr] / H_q / (n_win - jr) for jr in range(n_win)]
+        tot = sum(raw)
+        bw[l] = [x / tot for x in raw]
+    assert np.allclose(ts, bts, rtol=1e-12, atol=1e-15)
+    assert np.allclose(wt, bw, rtol=1e-12, atol=1e-15)
+
+
+def test_text_and_vision_mass_partition_every_row():
+    """Each causal row sums to 1 over text and vision keys, so G times the text
+    scores of Eq. 9 plus the TV statistic of Eq. 5 give H_q * n_win per layer."""
+    q, k, modality, pos, w = _rand_case(L=3, H_q=6, H_kv=3, d=7, seed=32)
+    ts, _ = oracle.text_scores_and_weights(q, k, modality, pos, 0.45, 3)
+    _, stat = oracle.twr_scores_tvb_stat(q, k, modality, pos, w, 0.45, 3)
+    G = 2
+    total = G * ts.sum(axis=(1, 2)) + stat
+    assert np.allclose(total, 6 * len(pos), rtol=1e-12)
+
+
+def test_eq7_uniform_attention_closed_form():
+    """Q = 0 gives A_ij = 1/(p_i + 1) on every visible key."""
+    q, k, modality, pos, _ = _rand_case(L=1, H_q=2, H_kv=1, seed=33)
+    q[:] = 0.0
+    ts, wt = oracle.text_scores_and_weights(q, k, modality, pos, 1.0, 1)
+    text = np.flatnonzero(modality == 0)
+    expect_ts = np.array([sum(1.0 / (p + 1) for p in pos if p >= t) for t in text])
+    assert np.allclose(ts[0, 0], expect_ts, rtol=1e-13)
+    n = len(pos)
+    raw = np.array([sum(1.0 / (pos[i] + 1) for i in range(j, n)) / (n - j) for j in range(n)])
+    assert np.allclose(wt[0], raw / raw.sum(), rtol=1e-13)
+
+
+def test_eq7_weights_normalised_and_single_row():
+    q, k, modality, pos, _ = _rand_case(L=2, seed=34)
+    _, wt = oracle.text_scores_and_weights(q, k, modality, pos, 0.9, 2)
+    assert np.allclose(wt.sum(axis=1), 1.0, rtol=1e-14) and np.all(wt > 0)
+    q1, k1, m1, p1, _ = _rand_case(L=2, n_win=1, seed=35)
+    _, w1 = oracle.text_scores_and_weights(q1, k1, m1, p1, 0.9, 2)
+    assert np.array_equal(w1, np.ones((2, 1)))
+
+
+def test_eq7_dominant_text_token_saturates():
+    """Every row attending almost only to the first window token (a dominant
+    text token) puts Eq. 7's weight on that row and its Eq. 9 score at n_win."""
+    q, k, modality, pos, _ = _rand_case(L=1, H_q=1, H_kv=1, d=6, seed=36)
+    u = np.zeros(6)
+    u[2] = 1.0
+    k[0, 0] = 0.0
+    k[0, 0, pos[0]] = u
+    q[0, 0] = 60.0 * u
+    ts, wt = oracle.text_scores_and_weights(q, k, modality, pos, 1.0, 1)
+    trank = int(np.count_nonzero(modality[:pos[0]] == 0))
+    assert abs(ts[0, 0, trank] - len(pos)) < 1e-9
+    assert wt[0, 0] > 1 - 1e-9
+
+
+def test_eq7_rejects_rows_on_vision_tokens():
+    q, k, modality, pos, _ = _rand_case(seed=37)
+    bad = pos.copy()
+    bad[0] = int(np.flatnonzero(modality == 1)[0])
+    bad.sort()
+    with pytest.raises(ValueError):
+        oracle.text_scores_and_weights(q, k, modality, bad, 1.0, 2)
+
+
+# ---------------------------------------------------------------- Eq. 10, both cases
+def _brute_select(vs, ts, b, modality, sinks, vision_basis=False):
+    vision = [j for j, m in enumerate(modality) if m == 1]
+    text = [j for j, m in enumerate(modality) if m == 0]
+    if vision_basis or b > len(text):
+        cand, sc, slots, keep = vision, vs, (b if vision_basis else b - len(text)), set(text)
+    else:
+        cand, sc, slots, keep = text, ts, b, set()
+    keep |= set(sinks)
+    free = [(-sc[r], j) for r, j in enumerate(cand) if j not in sinks]
+    slots = max(0, slots - sum(1 for j in cand if j in sinks))
+    for _, j in sorted(free)[:slots]:
+        keep.add(j)
+    return sorted(keep)
+
+
+@pytest.mark.parametrize("keep", [(0, 0), (4, 1), (2, 3)])
+def test_general_select_both_cases_brute_force(keep):
+    rng = np.random.default_rng(38)
+    modality = np.array([1, 1, 0, 0, 1, 0, 1, 1, 1, 0, 0, 1, 0, 1, 1, 0], np.uint8)
+    n_t, n_v = int((modality == 0).sum()), int((modality == 1).sum())
+    L, H = 6, 2
+    budgets = [0, 3, n_t, n_t + 1, n_t + 5, modality.size]
+    vs = rng.integers(0, 4, (L, H, n_v)).astype(np.float64)    # many ties
+    ts = rng.integers(0, 4, (L, H, n_t)).astype(np.float64)
+    sinks = list(oracle.sink_positions(modality.size, *keep))
+    off, idx = oracle.tpr_select_general(vs, ts, budgets, modality, *keep)
+    for l in range(L):
+        for g in range(H):
+            got = idx[off[l * H + g]:off[l * H + g + 1]].tolist()
+            assert got == _brute_select(vs[l, g], ts[l, g], budgets[l], modality, sinks)
+            if keep == (0, 0):
+                assert len(got) == budgets[l]
+            if budgets[l] > n_t:
+                assert set(np.flatnonzero(modality == 0)) <= set(got)
+            elif keep == (0, 0):
+                assert all(modality[j] == 0 for j in got)
+
+
+def test_general_select_vision_basis_is_tpr_select():
+    q, k, modality, pos, w = _rand_case(L=3, seed=39)
+    scores, stat = oracle.twr_scores_tvb_stat(q, k, modality, pos, w, 0.8, 2)
+    budgets = oracle.tvb_budgets(stat, 7, int((modality == 1).sum()))
+    a = oracle.tpr_select(scores, budgets, modality)
+    b = oracle.tpr_select_general(scores, None, budgets, modality, vision_basis=True)
+    assert np.array_equal(a[0], b[0]) and np.array_equal(a[1], b[1])
+
+
+def test_table4_memory_all_token_basis_mixed_layout():
+    """The main-text setting counts every KV in the ratio (Section 4.3): with
+    text and vision mixed, the all-token basis and Eq. 10 keep exactly
+    floor(r * N * L + 1/2) rows per head, reproducing Table 4's memory."""
+    path = os.path.join(os.path.dirname(__file__), "golden", "table4_kv_memory.txt")
+    rows = [line.split() for line in open(path) if line.strip() and not line.startswith("#")]
+    L, H_kv, d = 32, 32, 128
+    rng = np.random.default_rng(40)
+    for ctx, ratio, printed in rows:
+        ctx, ratio, printed = int(ctx), float(ratio), float(printed)
+        modality = np.zeros(ctx, np.uint8)
+        modality[35:35 + 576 * (ctx // 1000)] = 1                # a text prefix, images, a question
+        n_t, n_v = int((modality == 0).sum()), int((modality == 1).sum())
+        stat = 0.5 + rng.random(L)
+        total = oracle.all_budget_total(ratio, ctx, L)
+        budgets = oracle.tvb_budgets(stat, total, ctx)
+        assert sum(budgets) == total
+        vs = rng.random((L, 1, n_v))
+        ts = rng.random((L, 1, n_t))
+        offsets, _ = oracle.tpr_select_general(vs, ts, budgets, modality)
+        gib = H_kv * oracle.compacted_kv_bytes(offsets, d) / 2.0 ** 30
+        assert round(gib, 2) == printed, (ctx, ratio, gib)
+
+
+def test_evict_eq7_and_all_basis_tiny():
+    """End to end on the oracle: Eq. 7 weights feed Eq. 8; all-token budgets
+    sum to B and each head keeps b_l rows."""
+    rng = np.random.default_rng(41)
+    L, H_q, H_kv, d, n = 3, 4, 2, 8, 30
+    modality = np.zeros(n, np.uint8)
+    modality[4:22] = 1
+    pos = np.flatnonzero(modality == 0)[-6:]
+    qb = rng.integers(-2 ** 15, 2 ** 15, (L, H_q, pos.size, d)).astype(np.int16) & 0x3FFF
+    kb = rng.integers(-2 ** 15, 2 ** 15, (L, H_kv, n, d)).astype(np.int16) & 0x3FFF
+    vb = rng.integers(-2 ** 15, 2 ** 15, (L, H_kv, n, d)).astype(np.int16)
+    w = np.full((L, pos.size), 1.0 / pos.size)
+    r7 = oracle.evict(qb, kb, vb, modality, pos, w, 0.2, H_kv, weights="eq7")
+    q, k = oracle.widen_bf16(qb), oracle.widen_bf16(kb)
+    _, w7 = oracle.text_scores_and_weights(q, k, modality, pos, 1 / math.sqrt(d), H_kv)
+    s7, _ = oracle.twr_scores_tvb_stat(q, k, modality, pos, w7, 1 / math.sqrt(d), H_kv)
+    assert np.array_equal(r7["scores"], s7) and np.array_equal(r7["w"], w7)
+    for ratio in (0.1, 0.3, 0.9):
+        ra = oracle.evict(qb, kb, vb, modality, pos, w, ratio, H_kv, basis="all")
+        assert int(ra["budgets"].sum()) == oracle.all_budget_total(ratio, n, L)
+        for l in range(L):
+            for g in range(H_kv):
+                assert ra["offsets"][l * H_kv + g + 1] - ra["offsets"][l * H_kv + g] == ra["budgets"][l]
