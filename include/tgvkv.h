@@ -33,12 +33,28 @@
  * - Pointers to bf16 tensors, `workspace`, and the outputs k_out/v_out must be
  *   16-byte aligned.
  *
- * Budget basis.  The ratio r is the fraction of VISION KV kept over all layers
- * (the vision-only eviction setting of Appendix B.3, where the TPR policy keeps
- * every text KV): B_V = floor(r * N_v * L + 1/2) vision rows per head are
- * shared out over the layers.  Every KV head of layer l keeps the N_t text rows
- * and b_l vision rows, so the compacted cache holds
- * H_kv * (L * N_t + B_V) rows (tgvkv_retained_rows).
+ * Budget basis (desc->budget_basis).
+ * - TGVKV_BASIS_VISION (the default): the ratio r is the fraction of VISION KV
+ *   kept over all layers (the vision-only eviction setting of Appendix B.3,
+ *   where the TPR policy keeps every text KV): B_V = floor(r * N_v * L + 1/2)
+ *   vision rows per head are shared out over the layers.  Every KV head of
+ *   layer l keeps the N_t text rows and b_l vision rows, so the compacted
+ *   cache holds H_kv * (L * N_t + B_V) rows.
+ * - TGVKV_BASIS_ALL: r is the fraction of ALL KV kept (the main-text setting,
+ *   Section 4.3 / Table 4): B = floor(r * N * L + 1/2) rows per head are
+ *   shared out (cap N per layer), and Eq. 10 applies per layer: b_l > N_t keeps
+ *   every text row and the top (b_l - N_t) vision rows by the Eq. 8 score;
+ *   b_l <= N_t keeps the top b_l text rows by the Eq. 9 score and no vision.
+ * Sink tokens (desc->keep_first, desc->keep_last; Appendix A.2 keeps the first
+ * 4 and the last token for every method): always kept, each taking one slot of
+ * its own modality's part of the budget while slots remain.  Without sinks
+ * the cache holds exactly H_kv * (L * N_t + B_V) (vision basis) or H_kv * B
+ * (all-token basis) rows; sinks may add up to one row per sink per (l, g).
+ * tgvkv_retained_rows gives the capacity, offsets[L*H_kv] the rows written.
+ *
+ * Text weights (desc->weight_mode): TGVKV_WEIGHTS_GIVEN uses the caller's w~
+ * (Eq. 8); TGVKV_WEIGHTS_EQ7 makes tgvkv_evict derive w~ from the text-text
+ * attention by Eq. 7 (tgvkv_text_scores) and ignore `w`.
  */
 #ifndef TGVKV_H
 #define TGVKV_H
@@ -66,6 +82,12 @@ extern "C" {
 #define TGVKV_STATUS_TIMEOUT      0x20u /* a bounded on-chip wait gave up */
 #define TGVKV_STATUS_WEIGHT       0x40u /* a text weight is negative or not finite */
 
+/* ---- modes ------------------------------------------------------------ */
+#define TGVKV_BASIS_VISION  0   /* r counts vision KV; all text KV kept (default) */
+#define TGVKV_BASIS_ALL     1   /* r counts all KV; both cases of Eq. 10 */
+#define TGVKV_WEIGHTS_GIVEN 0   /* the caller's normalised text weights w~ (default) */
+#define TGVKV_WEIGHTS_EQ7   1   /* tgvkv_evict derives w~ by Eq. 7 */
+
 /* ---- problem description --------------------------------------------- */
 typedef struct tgvkv_desc {
     int32_t L;              /* decoder layers */
@@ -78,6 +100,10 @@ typedef struct tgvkv_desc {
     float   softmax_scale;  /* logits = softmax_scale * <q, k>; <= 0 means 1/sqrt(d) */
     int64_t w_layer_stride; /* floats between the weight rows of two layers; 0 = one
                                row shared by every layer */
+    int32_t budget_basis;   /* TGVKV_BASIS_VISION (0) or TGVKV_BASIS_ALL */
+    int32_t weight_mode;    /* TGVKV_WEIGHTS_GIVEN (0) or TGVKV_WEIGHTS_EQ7 (tgvkv_evict) */
+    int32_t keep_first;     /* sinks: the first keep_first positions are always kept */
+    int32_t keep_last;      /* ... and the last keep_last positions */
 } tgvkv_desc;
 
 /* Bytes of device workspace the calls below need for this problem. */
@@ -87,8 +113,15 @@ size_t tgvkv_workspace_size(const tgvkv_desc* desc);
  * layers (Eq. 5 splits it).  Returns -1 if desc or ratio (not in [0,1]) is bad. */
 int64_t tgvkv_vision_budget_total(const tgvkv_desc* desc, double ratio);
 
-/* Rows of the compacted cache, H_kv * (L * N_t + B_V); the capacity that idx,
- * k_out and v_out must have.  Returns -1 on bad arguments. */
+/* B of the descriptor's budget basis: B_V (vision basis) or
+ * floor(ratio * N * L + 1/2) rows of any modality (all-token basis).
+ * Returns -1 on bad arguments. */
+int64_t tgvkv_budget_total(const tgvkv_desc* desc, double ratio);
+
+/* Capacity of the compacted cache that idx, k_out and v_out must have:
+ * H_kv * (L * N_t + B_V) (vision basis) or H_kv * B (all-token basis), plus
+ * H_kv * L * (keep_first + keep_last) when there are sinks.  Returns -1 on bad
+ * arguments. */
 int64_t tgvkv_retained_rows(const tgvkv_desc* desc, double ratio);
 
 /* TWR scores and the TVB statistic (Eq. 2, 5, 6, 8).
@@ -113,12 +146,31 @@ int tgvkv_score(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
                 const uint8_t* modality, const int32_t* text_pos, const float* w,
                 float* scores, float* tvb_stat, void* workspace, void* stream);
 
+/* Text scores (Eq. 9) and derived text weights (Eq. 7).
+ *
+ * From the same causal attention rows as tgvkv_score (Eq. 2), sliced on the
+ * text keys (the text-text block A^(TT)):
+ *   text_scores[l][g][t] = (1/G) sum_{h in g} sum_i A_{l,h}[i, t]          (Eq. 9)
+ *   w_{l,j} = (1/H_q) sum_h sum_{i >= j} A_{l,h}[i, text_pos[j]] / (n_win - j)   (Eq. 7)
+ *   weights[l][j] = w_{l,j} / sum_j' w_{l,j'}      (the normalised w~)
+ * t runs over the text keys in position order; the rows i are the query rows
+ * (rows before key t see it as 0 through the causal mask).  Every query row
+ * must sit on a text token (else TGVKV_STATUS_TEXT_POS and a zero weight).
+ * text_scores: fp32 [L][H_kv][N_t] (output); weights: fp32 [L][n_win]
+ * (output; pass it to tgvkv_score as w with w_layer_stride = n_win).
+ * Other arguments as in tgvkv_score. */
+int tgvkv_text_scores(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* k,
+                      const uint8_t* modality, const int32_t* text_pos,
+                      float* text_scores, float* weights, void* workspace, void* stream);
+
 /* TVB layer budgets (Eq. 5, x = TV).  Splits B_V over the layers in proportion
  * to tvb_stat: b_l = floor(B_V * S_l / sum S) plus one leftover unit each for
  * the largest fractional parts (ties: lower layer); a layer above N_v is capped
  * at N_v and the rest re-split over the other layers; all-zero statistics give a
- * uniform split.  The quotients are computed in double on the device.
- * tvb_stat: fp32 [L]; budgets: int32 [L] (output, vision rows per KV head). */
+ * uniform split.  The quotients are computed in double on the device.  Under
+ * the all-token basis the same rule splits B with cap N.
+ * tvb_stat: fp32 [L]; budgets: int32 [L] (output, rows per KV head: vision rows
+ * under the vision basis, rows of any modality under the all-token basis). */
 int tgvkv_budget(const tgvkv_desc* desc, const float* tvb_stat, double ratio,
                  int32_t* budgets, void* workspace, void* stream);
 
@@ -133,6 +185,15 @@ int tgvkv_select(const tgvkv_desc* desc, const float* scores, const int32_t* bud
                  const uint8_t* modality, int64_t* offsets, int32_t* idx,
                  void* workspace, void* stream);
 
+/* TPR retention with every option of the descriptor (Eq. 10, both cases,
+ * sinks).  As tgvkv_select, plus text_scores: fp32 [L][H_kv][N_t] from
+ * tgvkv_text_scores, read for the layers with b_l <= N_t under the all-token
+ * basis (may be NULL under the vision basis).  tgvkv_select is this call with
+ * text_scores = NULL; it rejects the all-token basis. */
+int tgvkv_select_tpr(const tgvkv_desc* desc, const float* scores, const float* text_scores,
+                     const int32_t* budgets, const uint8_t* modality, int64_t* offsets,
+                     int32_t* idx, void* workspace, void* stream);
+
 /* Compaction: row r of set (l, g) of the CSR becomes
  *   k_out[r] = k[l][g][idx[r]],  v_out[r] = v[l][g][idx[r]]
  * as bit copies.  k, v: bf16 [L][H_kv][N][d]; k_out, v_out: bf16
@@ -142,7 +203,9 @@ int tgvkv_compact(const tgvkv_desc* desc, const uint16_t* k, const uint16_t* v,
                   uint16_t* k_out, uint16_t* v_out, void* workspace, void* stream);
 
 /* score -> budget -> select -> compact in one stream-ordered call with no host
- * synchronisation.  Arguments as in the four calls above. */
+ * synchronisation.  Arguments as in the four calls above.  With Eq. 7 weights
+ * or the all-token basis it first runs tgvkv_text_scores into the workspace
+ * (`w` is then ignored under TGVKV_WEIGHTS_EQ7). */
 int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* k,
                 const uint16_t* v, const uint8_t* modality, const int32_t* text_pos,
                 const float* w, double ratio,
@@ -154,7 +217,9 @@ int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
  * (introspection for callers that budget launches, e.g. inside a captured
  * graph; the paper has no counterpart): normally 2 (scores with the layer
  * budgets, then select + gather fused), 3 when the fused kernel's
- * shared-memory table does not fit (select and compact separately).  A problem
+ * shared-memory table does not fit (select and compact separately); 2 more
+ * (the text-key score pass and the Eq. 7 weights) with Eq. 7 weights or the
+ * all-token basis.  A problem
  * with no query rows zero-fills the scores with memsets and launches the
  * budget kernel in place of the score kernel.  Returns -1 on bad arguments. */
 int tgvkv_evict_launches(const tgvkv_desc* desc);

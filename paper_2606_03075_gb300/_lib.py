@@ -18,7 +18,13 @@ class Desc(ctypes.Structure):
     """Mirror of ``tgvkv_desc`` (include/tgvkv.h)."""
     _fields_ = [("L", c_int32), ("H_q", c_int32), ("H_kv", c_int32), ("d", c_int32),
                 ("N", c_int32), ("N_v", c_int32), ("n_win", c_int32),
-                ("softmax_scale", c_float), ("w_layer_stride", c_int64)]
+                ("softmax_scale", c_float), ("w_layer_stride", c_int64),
+                ("budget_basis", c_int32), ("weight_mode", c_int32),
+                ("keep_first", c_int32), ("keep_last", c_int32)]
+
+
+BASIS_VISION, BASIS_ALL = 0, 1
+WEIGHTS_GIVEN, WEIGHTS_EQ7 = 0, 1
 
 
 _P = ctypes.POINTER(Desc)
@@ -27,12 +33,17 @@ _P = ctypes.POINTER(Desc)
 SIGNATURES = {
     "tgvkv_workspace_size": (c_size_t, [_P]),
     "tgvkv_vision_budget_total": (c_int64, [_P, c_double]),
+    "tgvkv_budget_total": (c_int64, [_P, c_double]),
     "tgvkv_retained_rows": (c_int64, [_P, c_double]),
+    "tgvkv_text_scores": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                  c_void_p, c_void_p, c_void_p]),
     "tgvkv_score": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                             c_void_p, c_void_p, c_void_p, c_void_p]),
     "tgvkv_budget": (c_int, [_P, c_void_p, c_double, c_void_p, c_void_p, c_void_p]),
     "tgvkv_select": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                              c_void_p, c_void_p]),
+    "tgvkv_select_tpr": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                 c_void_p, c_void_p, c_void_p]),
     "tgvkv_compact": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                               c_void_p, c_void_p, c_void_p]),
     "tgvkv_evict": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,

@@ -28,15 +28,27 @@ class TgvkvError(RuntimeError):
         self.code = code
 
 
-def make_desc(L, H_q, H_kv, d, N, N_v, n_win, softmax_scale=0.0, w_layer_stride=None) -> Desc:
-    """A problem descriptor; w_layer_stride defaults to n_win (one weight row per layer)."""
+BASIS = {"vision": _lib.BASIS_VISION, "all": _lib.BASIS_ALL}
+WEIGHTS = {"given": _lib.WEIGHTS_GIVEN, "eq7": _lib.WEIGHTS_EQ7}
+
+
+def make_desc(L, H_q, H_kv, d, N, N_v, n_win, softmax_scale=0.0, w_layer_stride=None,
+              basis="vision", weights="given", keep_first=0, keep_last=0) -> Desc:
+    """A problem descriptor; w_layer_stride defaults to n_win (one weight row per layer).
+
+    basis: "vision" (r counts vision KV, every text KV kept) or "all" (r counts
+    every KV, both cases of Eq. 10); weights: "given" (the caller's w~) or
+    "eq7" (tgvkv_evict derives w~ by Eq. 7); keep_first / keep_last: sinks."""
     return Desc(L=L, H_q=H_q, H_kv=H_kv, d=d, N=N, N_v=N_v, n_win=n_win,
                 softmax_scale=float(softmax_scale),
-                w_layer_stride=n_win if w_layer_stride is None else w_layer_stride)
+                w_layer_stride=n_win if w_layer_stride is None else w_layer_stride,
+                budget_basis=BASIS[basis], weight_mode=WEIGHTS[weights],
+                keep_first=keep_first, keep_last=keep_last)
 
 
-def desc_for_workload(wl, softmax_scale=0.0) -> Desc:
-    return make_desc(wl.L, wl.H_q, wl.H_kv, wl.d, wl.N, wl.N_v, wl.n_win, softmax_scale)
+def desc_for_workload(wl, softmax_scale=0.0, **options) -> Desc:
+    return make_desc(wl.L, wl.H_q, wl.H_kv, wl.d, wl.N, wl.N_v, wl.n_win, softmax_scale,
+                     **options)
 
 
 def _stream(stream):
@@ -82,6 +94,13 @@ def tgvkv_vision_budget_total(desc: Desc, ratio: float) -> int:
     return int(n)
 
 
+def tgvkv_budget_total(desc: Desc, ratio: float) -> int:
+    n = _lib.load().tgvkv_budget_total(ctypes.byref(desc), float(ratio))
+    if n < 0:
+        raise TgvkvError(-1, "tgvkv_budget_total")
+    return int(n)
+
+
 def tgvkv_retained_rows(desc: Desc, ratio: float) -> int:
     n = _lib.load().tgvkv_retained_rows(ctypes.byref(desc), float(ratio))
     if n < 0:
@@ -118,6 +137,20 @@ def tgvkv_score(desc, q_text, k, modality, text_pos, w, scores, tvb_stat, ws, st
         _stream(stream)), "tgvkv_score")
 
 
+def tgvkv_text_scores(desc, q_text, k, modality, text_pos, text_scores, weights, ws, stream=None):
+    L, Hq, Hkv, d, N, nw = desc.L, desc.H_q, desc.H_kv, desc.d, desc.N, desc.n_win
+    _check(_lib.load().tgvkv_text_scores(
+        ctypes.byref(desc),
+        _ptr(q_text, _BF16_LIKE, L * Hq * nw * d, "q_text"),
+        _ptr(k, _BF16_LIKE, L * Hkv * N * d, "k"),
+        _ptr(modality, (torch.uint8,), N, "modality"),
+        _ptr(text_pos, (torch.int32,), nw, "text_pos"),
+        _ptr(text_scores, (torch.float32,), L * Hkv * (N - desc.N_v), "text_scores"),
+        _ptr(weights, (torch.float32,), L * nw, "weights"),
+        _ptr(ws, (torch.uint8,), tgvkv_workspace_size(desc), "workspace"),
+        _stream(stream)), "tgvkv_text_scores")
+
+
 def tgvkv_budget(desc, tvb_stat, ratio, budgets, ws, stream=None):
     _check(_lib.load().tgvkv_budget(
         ctypes.byref(desc),
@@ -138,6 +171,20 @@ def tgvkv_select(desc, scores, budgets, modality, offsets, idx, ws, stream=None)
         _ptr(idx, (torch.int32,), 0, "idx"),
         _ptr(ws, (torch.uint8,), tgvkv_workspace_size(desc), "workspace"),
         _stream(stream)), "tgvkv_select")
+
+
+def tgvkv_select_tpr(desc, scores, text_scores, budgets, modality, offsets, idx, ws, stream=None):
+    LH = desc.L * desc.H_kv
+    _check(_lib.load().tgvkv_select_tpr(
+        ctypes.byref(desc),
+        _ptr(scores, (torch.float32,), LH * desc.N_v, "scores"),
+        _ptr(text_scores, (torch.float32,), LH * (desc.N - desc.N_v), "text_scores"),
+        _ptr(budgets, (torch.int32,), desc.L, "budgets"),
+        _ptr(modality, (torch.uint8,), desc.N, "modality"),
+        _ptr(offsets, (torch.int64,), LH + 1, "offsets"),
+        _ptr(idx, (torch.int32,), 0, "idx"),
+        _ptr(ws, (torch.uint8,), tgvkv_workspace_size(desc), "workspace"),
+        _stream(stream)), "tgvkv_select_tpr")
 
 
 def tgvkv_compact(desc, k, v, offsets, idx, k_out, v_out, ws, stream=None):

@@ -37,6 +37,10 @@ bool aligned16(const void* ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u
 
 size_t round_up(size_t x) { return (x + 255) & ~size_t(255); }
 
+// tgvkv_evict needs the Eq. 9 text scores: for Eq. 7 weights, or for case
+// b_l <= N_t of Eq. 10 under the all-token basis.
+bool needs_text_pass(const Problem& p) { return p.weights_eq7 || p.basis == TGVKV_BASIS_ALL; }
+
 WsLayout layout_of(const Problem& p) {
     WsLayout w;
     size_t o = 0;
@@ -45,7 +49,14 @@ WsLayout layout_of(const Problem& p) {
     w.stat_part = o;   o += round_up(sizeof(float) * (size_t)p.L * p.H_kv * (p.T > 0 ? p.T : 1));
     w.stat_head = o;   o += round_up(sizeof(float) * (size_t)p.L * p.H_kv);
     w.score_part = o;
-    if (p.T > 1) o += round_up(sizeof(float) * (size_t)p.L * p.H_kv * p.T * (size_t)p.N_v);
+    const size_t keyset = (size_t)(p.N_v > p.N_t ? p.N_v : p.N_t);
+    if (p.T > 1) o += round_up(sizeof(float) * (size_t)p.L * p.H_kv * p.T * keyset);
+    w.stat_text = o;   o += round_up(sizeof(float) * (size_t)p.L);
+    w.text_scores = w.weights = 0;
+    if (needs_text_pass(p)) {
+        w.text_scores = o; o += round_up(sizeof(float) * (size_t)p.L * p.H_kv * (p.N_t > 0 ? p.N_t : 1));
+        w.weights = o;     o += round_up(sizeof(float) * (size_t)p.L * (p.n_win > 0 ? p.n_win : 1));
+    }
     w.total = o;
     return w;
 }
@@ -90,6 +101,18 @@ int make_problem(const tgvkv_desc* d, Problem* p) {
     const double scale = d->softmax_scale > 0.f ? (double)d->softmax_scale : 1.0 / sqrt((double)d->d);
     p->scale_log2 = (float)(scale * 1.4426950408889634);  // log2(e)
     p->w_stride = (long long)d->w_layer_stride;
+    if (d->budget_basis != TGVKV_BASIS_VISION && d->budget_basis != TGVKV_BASIS_ALL)
+        return fail(TGVKV_ERR_INVALID_ARG, "budget_basis=%d unknown", d->budget_basis);
+    if (d->weight_mode != TGVKV_WEIGHTS_GIVEN && d->weight_mode != TGVKV_WEIGHTS_EQ7)
+        return fail(TGVKV_ERR_INVALID_ARG, "weight_mode=%d unknown", d->weight_mode);
+    if (d->keep_first < 0 || d->keep_last < 0)
+        return fail(TGVKV_ERR_INVALID_ARG, "keep_first=%d / keep_last=%d < 0", d->keep_first,
+                    d->keep_last);
+    p->basis = d->budget_basis;
+    p->weights_eq7 = d->weight_mode == TGVKV_WEIGHTS_EQ7;
+    p->keep_first = d->keep_first < d->N ? d->keep_first : d->N;
+    p->keep_last = d->keep_last < d->N ? d->keep_last : d->N;
+    p->keys_text = 0;
     return TGVKV_OK;
 }
 
@@ -99,12 +122,34 @@ int check_ratio(double ratio) {
     return TGVKV_OK;
 }
 
-long long budget_total(const Problem& p, double ratio) {
+long long vision_budget_total(const Problem& p, double ratio) {
     return (long long)floor(ratio * (double)((long long)p.N_v * p.L) + 0.5);
 }
 
+// B: rows per head over all layers that the budget split shares out --
+// vision rows (vision basis) or rows of any modality (all-token basis).
+long long budget_total(const Problem& p, double ratio) {
+    if (p.basis == TGVKV_BASIS_ALL) return (long long)floor(ratio * (double)((long long)p.N * p.L) + 0.5);
+    return vision_budget_total(p, ratio);
+}
+
+// The cap of one layer's budget in the split.
+int budget_cap(const Problem& p) { return p.basis == TGVKV_BASIS_ALL ? p.N : p.N_v; }
+
+// Sink positions (at most N).
+int n_sinks(const Problem& p) {
+    const int both = p.keep_first + p.keep_last;
+    return both < p.N ? both : p.N;
+}
+
+// Capacity of the compacted cache.  Exact without sinks: H_kv * (L * N_t + B_V)
+// (vision basis) or H_kv * B (all-token basis).  A sink can add one row above a
+// layer's budget, so sinks add at most H_kv * L * (keep_first + keep_last).
 long long retained_rows(const Problem& p, double ratio) {
-    return (long long)p.H_kv * ((long long)p.L * p.N_t + budget_total(p, ratio));
+    const long long base = p.basis == TGVKV_BASIS_ALL
+                               ? budget_total(p, ratio)
+                               : (long long)p.L * p.N_t + budget_total(p, ratio);
+    return (long long)p.H_kv * (base + (long long)p.L * n_sinks(p));
 }
 
 #define REQUIRE_PTR(ptr, name, need16)                                                   \
@@ -127,13 +172,41 @@ int do_score(const Problem& p, const uint16_t* q, const uint16_t* k, const uint8
     return e == cudaSuccess ? TGVKV_OK : cuda_fail(e, "score launch");
 }
 
+// The problem of the text-key pass (Eq. 9): the score kernel with the key set
+// and its size swapped to the text keys.
+Problem text_problem(const Problem& p) {
+    Problem t = p;
+    t.keys_text = 1;
+    t.N_v = p.N_t;
+    t.N_t = p.N_v;
+    return t;
+}
+
+// Eq. 9 text scores and Eq. 7 weights: the text-key score pass, then the
+// per-layer weights.  stat_scratch takes the pass's (unused) statistic.
+int do_text_scores(const Problem& p, const uint16_t* q, const uint16_t* k, const uint8_t* modality,
+                   const int32_t* text_pos, float* text_scores, float* weights, float* stat_scratch,
+                   void* ws, cudaStream_t st) {
+    const WsLayout lay = layout_of(p);
+    const Problem tp = text_problem(p);
+    cudaError_t e = launch_score(tp, q, k, modality, text_pos, nullptr, text_scores, stat_scratch,
+                                 static_cast<char*>(ws), lay, -1, nullptr, st);
+    if (e != cudaSuccess) return cuda_fail(e, "text-key score launch");
+    if (weights) {
+        e = launch_eq7_weights(p, text_scores, modality, text_pos, weights, status_of(ws, lay), st);
+        if (e != cudaSuccess) return cuda_fail(e, "Eq. 7 weights launch");
+    }
+    return TGVKV_OK;
+}
+
 int check_score_args(const Problem& p, const uint16_t* q, const uint16_t* k,
                      const uint8_t* modality, const int32_t* text_pos, const float* w,
-                     const float* scores, const float* tvb_stat, const void* ws) {
+                     const float* scores, const float* tvb_stat, const void* ws,
+                     bool need_w = true) {
     if (p.n_win > 0) {
         REQUIRE_PTR(q, "q_text", true);
         REQUIRE_PTR(text_pos, "text_pos", false);
-        REQUIRE_PTR(w, "w", false);
+        if (need_w) REQUIRE_PTR(w, "w", false);
     }
     REQUIRE_PTR(k, "k", true);
     REQUIRE_PTR(modality, "modality", false);
@@ -162,6 +235,12 @@ int64_t tgvkv_vision_budget_total(const tgvkv_desc* desc, double ratio) {
     return budget_total(p, ratio);
 }
 
+int64_t tgvkv_budget_total(const tgvkv_desc* desc, double ratio) {
+    Problem p{};
+    if (make_problem(desc, &p) != TGVKV_OK || check_ratio(ratio) != TGVKV_OK) return -1;
+    return budget_total(p, ratio);
+}
+
 int64_t tgvkv_retained_rows(const tgvkv_desc* desc, double ratio) {
     Problem p{};
     if (make_problem(desc, &p) != TGVKV_OK || check_ratio(ratio) != TGVKV_OK) return -1;
@@ -181,6 +260,28 @@ int tgvkv_score(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
     return rc ? rc : ok();
 }
 
+int tgvkv_text_scores(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* k,
+                      const uint8_t* modality, const int32_t* text_pos, float* text_scores,
+                      float* weights, void* workspace, void* stream) {
+    Problem p{};
+    int rc = make_problem(desc, &p);
+    if (rc) return rc;
+    if (p.n_win > 0) {
+        REQUIRE_PTR(q_text, "q_text", true);
+        REQUIRE_PTR(text_pos, "text_pos", false);
+        REQUIRE_PTR(weights, "weights", false);
+    }
+    REQUIRE_PTR(k, "k", true);
+    REQUIRE_PTR(modality, "modality", false);
+    if (p.N_t > 0) REQUIRE_PTR(text_scores, "text_scores", false);
+    REQUIRE_PTR(workspace, "workspace", true);
+    const WsLayout lay = layout_of(p);
+    float* scratch = reinterpret_cast<float*>(static_cast<char*>(workspace) + lay.stat_text);
+    rc = do_text_scores(p, q_text, k, modality, text_pos, text_scores, p.n_win > 0 ? weights : nullptr,
+                        scratch, workspace, static_cast<cudaStream_t>(stream));
+    return rc ? rc : ok();
+}
+
 int tgvkv_budget(const tgvkv_desc* desc, const float* tvb_stat, double ratio, int32_t* budgets,
                  void* workspace, void* stream) {
     Problem p{};
@@ -196,22 +297,33 @@ int tgvkv_budget(const tgvkv_desc* desc, const float* tvb_stat, double ratio, in
     return e == cudaSuccess ? ok() : cuda_fail(e, "budget launch");
 }
 
-int tgvkv_select(const tgvkv_desc* desc, const float* scores, const int32_t* budgets,
-                 const uint8_t* modality, int64_t* offsets, int32_t* idx, void* workspace,
-                 void* stream) {
+int tgvkv_select_tpr(const tgvkv_desc* desc, const float* scores, const float* text_scores,
+                     const int32_t* budgets, const uint8_t* modality, int64_t* offsets,
+                     int32_t* idx, void* workspace, void* stream) {
     Problem p{};
     int rc = make_problem(desc, &p);
     if (rc) return rc;
     if (p.N_v > 0) REQUIRE_PTR(scores, "scores", false);
+    if (p.basis == TGVKV_BASIS_ALL && p.N_t > 0) REQUIRE_PTR(text_scores, "text_scores", false);
     REQUIRE_PTR(budgets, "budgets", false);
     REQUIRE_PTR(modality, "modality", false);
     REQUIRE_PTR(offsets, "offsets", false);
     REQUIRE_PTR(idx, "idx", false);
     REQUIRE_PTR(workspace, "workspace", true);
     const WsLayout lay = layout_of(p);
-    cudaError_t e = launch_select(p, scores, budgets, modality, offsets, idx,
+    cudaError_t e = launch_select(p, scores, text_scores, budgets, modality, offsets, idx,
                                   status_of(workspace, lay), static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? ok() : cuda_fail(e, "select launch");
+}
+
+int tgvkv_select(const tgvkv_desc* desc, const float* scores, const int32_t* budgets,
+                 const uint8_t* modality, int64_t* offsets, int32_t* idx, void* workspace,
+                 void* stream) {
+    if (desc && desc->budget_basis == TGVKV_BASIS_ALL)
+        return fail(TGVKV_ERR_INVALID_ARG,
+                    "the all-token basis needs the text scores: use tgvkv_select_tpr");
+    return tgvkv_select_tpr(desc, scores, nullptr, budgets, modality, offsets, idx, workspace,
+                            stream);
 }
 
 int tgvkv_compact(const tgvkv_desc* desc, const uint16_t* k, const uint16_t* v,
@@ -244,7 +356,8 @@ int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
     int rc = make_problem(desc, &p);
     if (rc) return rc;
     if ((rc = check_ratio(ratio))) return rc;
-    rc = check_score_args(p, q_text, k, modality, text_pos, w, scores, tvb_stat, workspace);
+    rc = check_score_args(p, q_text, k, modality, text_pos, w, scores, tvb_stat, workspace,
+                          !p.weights_eq7);
     if (rc) return rc;
     REQUIRE_PTR(v, "v", true);
     REQUIRE_PTR(budgets, "budgets", false);
@@ -255,17 +368,32 @@ int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     const WsLayout lay = layout_of(p);
     uint32_t* status = status_of(workspace, lay);
+    char* wsb = static_cast<char*>(workspace);
+    float* text_scores = nullptr;
+    if (needs_text_pass(p)) {
+        // Eq. 9 text scores (and Eq. 7 weights) into the workspace first
+        text_scores = reinterpret_cast<float*>(wsb + lay.text_scores);
+        float* wts = p.weights_eq7 ? reinterpret_cast<float*>(wsb + lay.weights) : nullptr;
+        rc = do_text_scores(p, q_text, k, modality, text_pos, text_scores, p.n_win > 0 ? wts : nullptr,
+                            reinterpret_cast<float*>(wsb + lay.stat_text), workspace, st);
+        if (rc) return rc;
+    }
+    Problem ps = p;
+    const float* w_used = w;
+    if (p.weights_eq7) {
+        w_used = reinterpret_cast<const float*>(wsb + lay.weights);
+        ps.w_stride = p.n_win;
+    }
     // the score kernel's last CTA also derives the layer budgets
-    cudaError_t e = launch_score(p, q_text, k, modality, text_pos, w, scores, tvb_stat,
-                                 static_cast<char*>(workspace), lay, budget_total(p, ratio), budgets,
-                                 st);
+    cudaError_t e = launch_score(ps, q_text, k, modality, text_pos, w_used, scores, tvb_stat,
+                                 wsb, lay, budget_total(p, ratio), budgets, st);
     if (e != cudaSuccess) return cuda_fail(e, "score launch");
     if (score_launches(p) == 0) {   // no score kernel ran: split the (zero) statistic here
         e = launch_budget(p, tvb_stat, budget_total(p, ratio), budgets, status, st);
         if (e != cudaSuccess) return cuda_fail(e, "budget launch");
     }
-    e = launch_select_compact(p, scores, budgets, modality, offsets, idx, k, v, k_out, v_out,
-                              retained_rows(p, ratio), status, st);
+    e = launch_select_compact(p, scores, text_scores, budgets, modality, offsets, idx, k, v, k_out,
+                              v_out, retained_rows(p, ratio), status, st);
     if (e != cudaSuccess) return cuda_fail(e, "select/compact launch");
     return ok();
 }
@@ -273,7 +401,8 @@ int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
 int tgvkv_evict_launches(const tgvkv_desc* desc) {
     Problem p{};
     if (make_problem(desc, &p) != TGVKV_OK) return -1;
-    return (score_launches(p) == 0 ? 1 : score_launches(p)) + select_compact_launches(p);
+    const int text = needs_text_pass(p) ? score_launches(p) + (p.weights_eq7 && p.n_win > 0 ? 1 : 0) : 0;
+    return text + (score_launches(p) == 0 ? 1 : score_launches(p)) + select_compact_launches(p);
 }
 
 int tgvkv_workspace_init(const tgvkv_desc* desc, void* workspace, void* stream) {

@@ -15,7 +15,19 @@ struct Problem {
     int T;                 // 128-row tiles per KV head: ceil(R / 128)
     float scale_log2;      // softmax_scale * log2(e): logits in base-2 units
     long long w_stride;    // floats between the weight rows of two layers
+    int basis;             // TGVKV_BASIS_VISION or TGVKV_BASIS_ALL
+    int weights_eq7;       // tgvkv_evict derives w~ by Eq. 7
+    int keep_first, keep_last;   // sink tokens, clipped to [0, N]
+    // Score kernel only: the key set of pass B.  0 = vision keys (Eq. 8, row
+    // weights w~); 1 = text keys with unit row weights (Eq. 9).  N_v then
+    // holds the size of that key set, N_t; the launcher sets both.
+    int keys_text;
 };
+
+// Sinks among the positions 0..N-1: the first keep_first and the last keep_last.
+__host__ __device__ inline bool is_sink(const Problem& p, int j) {
+    return j < p.keep_first || j >= p.N - p.keep_last;
+}
 
 // Workspace layout (byte offsets into the caller's buffer).
 struct WsLayout {
@@ -23,7 +35,11 @@ struct WsLayout {
     size_t tickets;     // uint32 [ticket_words]: completion counters (heads), kernel counters
     size_t stat_part;   // float [L*H_kv*T]: TV mass of one row tile
     size_t stat_head;   // float [L*H_kv]: TV mass of one KV head
-    size_t score_part;  // float [L*H_kv*T*N_v]: scores of one row tile (T > 1)
+    size_t score_part;  // float [L*H_kv*T*max(N_v,N_t)]: scores of one row tile (T > 1)
+    // tgvkv_evict with Eq. 7 weights or the all-token basis only (0 otherwise):
+    size_t text_scores; // float [L*H_kv*N_t]: Eq. 9 scores
+    size_t weights;     // float [L*n_win]: Eq. 7 weights
+    size_t stat_text;   // float [L]: the text-key pass's (unused) statistic
     size_t total;
 };
 

@@ -19,22 +19,31 @@ cudaError_t launch_score(const Problem& p, const uint16_t* q, const uint16_t* k,
                          float* scores, float* tvb_stat, char* ws, const WsLayout& lay,
                          long long budget_total, int32_t* budgets, cudaStream_t stream);
 
+// TVB split of `total` (budget.cu); the cap is N_v (vision basis) or N.
 cudaError_t launch_budget(const Problem& p, const float* tvb_stat, long long total,
                           int32_t* budgets, uint32_t* status, cudaStream_t stream);
 
-cudaError_t launch_select(const Problem& p, const float* scores, const int32_t* budgets,
-                          const uint8_t* modality, int64_t* offsets, int32_t* idx,
-                          uint32_t* status, cudaStream_t stream);
+// TPR selection (select.cu).  text_scores (Eq. 9) is read only under the
+// all-token basis for layers with b_l <= N_t.
+cudaError_t launch_select(const Problem& p, const float* scores, const float* text_scores,
+                          const int32_t* budgets, const uint8_t* modality, int64_t* offsets,
+                          int32_t* idx, uint32_t* status, cudaStream_t stream);
 
 // select + gather fused (tgvkv_evict): one CTA per (layer, KV head) selects
 // its set and gathers its rows; falls back to the separate select and compact
 // kernels when the keys and retained rows of a head do not fit in shared
 // memory.
-cudaError_t launch_select_compact(const Problem& p, const float* scores, const int32_t* budgets,
-                                  const uint8_t* modality, int64_t* offsets, int32_t* idx,
-                                  const uint16_t* k, const uint16_t* v, uint16_t* k_out,
-                                  uint16_t* v_out, long long capacity_rows, uint32_t* status,
-                                  cudaStream_t stream);
+cudaError_t launch_select_compact(const Problem& p, const float* scores, const float* text_scores,
+                                  const int32_t* budgets, const uint8_t* modality,
+                                  int64_t* offsets, int32_t* idx, const uint16_t* k,
+                                  const uint16_t* v, uint16_t* k_out, uint16_t* v_out,
+                                  long long capacity_rows, uint32_t* status, cudaStream_t stream);
+
+// Eq. 7 weights from the Eq. 9 text scores (text.cu): weights[l][j] for the
+// query rows, L1-normalised per layer.
+cudaError_t launch_eq7_weights(const Problem& p, const float* text_scores, const uint8_t* modality,
+                               const int32_t* text_pos, float* weights, uint32_t* status,
+                               cudaStream_t stream);
 
 // Kernels launch_score / launch_select_compact launch for p.
 int score_launches(const Problem& p);

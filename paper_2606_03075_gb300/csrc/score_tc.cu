@@ -40,6 +40,10 @@
 // the softmax, four per TMEM lane quarter.  Every wait is bounded (about 1 s
 // of SM cycles); a timeout sets TGVKV_STATUS_TIMEOUT and the CTA unwinds.
 //
+// With Problem::keys_text set, pass B runs over the text keys with unit row
+// weights (c_i = 1 / (G Z_i)): the text scores of Eq. 9.  The launcher then
+// passes N_t as the key-set size in N_v.
+//
 // Results do not depend on the schedule: every key's pass-B sum is two
 // partial sums added onto zero (the same in either order); the row tiles of a
 // head write partial score rows that the last pair to finish adds in tile
@@ -419,7 +423,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
 #pragma unroll
         for (int wd = 0; wd < 4; ++wd) {
             const int j = kt * BN + wd * 32 + lane;
-            const unsigned m = __ballot_sync(~0u, j < p.N && modality[j] != 0);
+            // the key set of pass B: vision keys, or text keys (Eq. 9)
+            const unsigned m = __ballot_sync(~0u, j < p.N && (modality[j] != 0) != (p.keys_text != 0));
             if (lane == 0) {
                 s.vmask[kt][wd] = m;
                 s.vq[kt][wd] = cnt;              // within the tile, for now
@@ -715,10 +720,14 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
                     const int wi_row = (t_row + row) % p.n_win;
                     pos = text_pos[wi_row];
                     if (pos < 0 || pos >= p.N) pos = -1;
-                    wr = w[(long long)Item::pick(itm.l, part) * p.w_stride + wi_row];
-                    if (!(wr >= 0.f) || isinf(wr)) {
-                        raise_status(status, TGVKV_STATUS_WEIGHT);
-                        wr = 0.f;
+                    if (p.keys_text) {
+                        wr = 1.f;   // Eq. 9: unweighted column sums
+                    } else {
+                        wr = w[(long long)Item::pick(itm.l, part) * p.w_stride + wi_row];
+                        if (!(wr >= 0.f) || isinf(wr)) {
+                            raise_status(status, TGVKV_STATUS_WEIGHT);
+                            wr = 0.f;
+                        }
                     }
                 }
                 s.row_pos[rs][ln] = pos;
@@ -989,7 +998,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
             // the layer budgets of Eq. 5, with the now idle K ring as scratch
             __syncthreads();
             static_assert(sizeof(BudgetScratch) <= sizeof(s.k), "budget scratch in the K ring");
-            tvb_budget_block(tvb_stat, p.L, budget_total, p.N_v, budgets, status,
+            tvb_budget_block(tvb_stat, p.L, budget_total, p.basis == TGVKV_BASIS_ALL ? p.N : p.N_v,
+                             budgets, status,
                              *reinterpret_cast<BudgetScratch*>(&s.k[0][0][0]));
         }
         if (tid == 0) *exit_counter = 0u;

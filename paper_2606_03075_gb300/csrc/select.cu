@@ -1,4 +1,5 @@
-// TPR retention (Eq. 10, case b_l > N_t, vision budget b_l): one CTA per
+// TPR retention (Eq. 10).  The hot path (vision basis, no sinks) is the case
+// b_l > N_t with the vision budget b_l: one CTA per
 // (layer, KV head) keeps every text position and the b_l vision positions of
 // highest score, ties to the lower position, in ascending position order --
 // and, in the fused form used by tgvkv_evict, gathers the retained K and V
@@ -407,6 +408,274 @@ tpr_select_warp_kernel(Problem p, const float* __restrict__ scores,
     }
 }
 
+// ---- the general form: both cases of Eq. 10 and sink tokens (any basis).
+// Per layer the case is chosen by b_l: under the all-token basis b_l > N_t
+// ranks the vision keys by the Eq. 8 score on top of every text key, and
+// b_l <= N_t ranks the text keys by the Eq. 9 score with no vision key;
+// under the vision basis the first case holds with b_l vision slots.  Sinks
+// are always kept; a sink of the ranked modality takes one slot (its key is
+// set to 0, below every score's key, so the radix select never picks it).
+struct TprCase {
+    bool vision;   // the ranked candidates are the vision keys
+    int slots;     // candidates chosen by rank (sinks excluded)
+    int len;       // retained rows of each head of the layer
+};
+
+__host__ __device__ inline TprCase tpr_case(const Problem& p, int b, int sink_v, int sink_t) {
+    TprCase c;
+    const bool all = p.basis == TGVKV_BASIS_ALL;
+    c.vision = !all || b > p.N_t;
+    const int n_cand = c.vision ? p.N_v : p.N_t;
+    const int sink_c = c.vision ? sink_v : sink_t;
+    int slots = (all && c.vision) ? b - p.N_t : b;
+    slots -= sink_c;
+    slots = slots < 0 ? 0 : (slots > n_cand - sink_c ? n_cand - sink_c : slots);
+    c.slots = slots;
+    c.len = (c.vision ? p.N_t + sink_v : sink_v + sink_t) + slots;
+    return c;
+}
+
+__host__ __device__ inline int budget_cap_of(const Problem& p) {
+    return p.basis == TGVKV_BASIS_ALL ? p.N : p.N_v;
+}
+
+__host__ __device__ inline size_t select_general_smem(const Problem& p, bool compact) {
+    const size_t keyset = (size_t)(p.N_v > p.N_t ? p.N_v : p.N_t);
+    return sizeof(uint32_t) * keyset + (compact ? sizeof(int) * (size_t)p.N : 0) +
+           (((size_t)p.N + 15) & ~size_t(15));
+}
+
+template <bool COMPACT, int VPR>
+__global__ void __launch_bounds__(kThreads)
+tpr_select_general_kernel(Problem p, const float* __restrict__ scores,
+                          const float* __restrict__ text_scores,
+                          const int32_t* __restrict__ budgets, const uint8_t* __restrict__ modality_g,
+                          int64_t* __restrict__ offsets, int32_t* __restrict__ idx,
+                          const uint4* __restrict__ k, const uint4* __restrict__ v,
+                          uint4* __restrict__ k_out, uint4* __restrict__ v_out,
+                          uint32_t* __restrict__ status) {
+    extern __shared__ __align__(16) unsigned char dyn_raw[];
+    const size_t keyset = (size_t)(p.N_v > p.N_t ? p.N_v : p.N_t);
+    uint32_t* keys = reinterpret_cast<uint32_t*>(dyn_raw);          // [candidates]
+    int* rows = reinterpret_cast<int*>(keys + keyset);             // [len] (gather form)
+    uint8_t* modality = reinterpret_cast<uint8_t*>(dyn_raw) + sizeof(uint32_t) * keyset +
+                        (COMPACT ? sizeof(int) * (size_t)p.N : 0);   // [N]
+    __shared__ int hist[256];
+    __shared__ int scan_buf[33];
+    __shared__ uint32_t s_prefix;
+    __shared__ int s_kk, s_sink_v, s_sink_t;
+    __shared__ long long s_off;
+
+    const int lg = blockIdx.x, l = lg / p.H_kv, g = lg % p.H_kv;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    if (tid == 0) {
+        s_sink_v = 0;
+        s_sink_t = 0;
+    }
+    __syncthreads();
+    int sv = 0, st = 0;
+    for (int j = tid; j < p.N; j += kThreads) {
+        const uint8_t m = __ldg(modality_g + j);
+        modality[j] = m;
+        if (is_sink(p, j)) (m != 0 ? sv : st) += 1;
+    }
+    if (sv) atomicAdd(&s_sink_v, sv);
+    if (st) atomicAdd(&s_sink_t, st);
+    __syncthreads();
+    const int sink_v = s_sink_v, sink_t = s_sink_t;
+    const int cap = budget_cap_of(p);
+    int b = budgets[l];
+    if (b < 0 || b > cap) {
+        if (tid == 0) raise_status(status, TGVKV_STATUS_BUDGET);
+        b = b < 0 ? 0 : cap;
+    }
+    const TprCase c = tpr_case(p, b, sink_v, sink_t);
+    const int len = c.len;
+    if (tid == 0) {
+        long long off = 0;
+        for (int m = 0; m < l; ++m) {
+            int bm = budgets[m];
+            bm = bm < 0 ? 0 : (bm > cap ? cap : bm);
+            off += (long long)p.H_kv * tpr_case(p, bm, sink_v, sink_t).len;
+        }
+        off += (long long)g * len;
+        s_off = off;
+        offsets[lg] = off;
+        if (lg == p.L * p.H_kv - 1) offsets[lg + 1] = off + len;
+    }
+    const int n_cand = c.vision ? p.N_v : p.N_t;
+    const uint8_t cand_mod = c.vision ? 1 : 0;
+    const float* sc = c.vision ? scores + (size_t)lg * p.N_v : text_scores + (size_t)lg * p.N_t;
+    for (int i = tid; i < n_cand; i += kThreads) keys[i] = float_order_key(__ldg(sc + i));
+    __syncthreads();
+
+    // ---- candidate ranks of each thread's contiguous position range; sinks get key 0
+    const int per = (p.N + kThreads - 1) / kThreads;
+    const int j0 = min(p.N, tid * per), j1 = min(p.N, j0 + per);
+    int nc = 0;
+    for (int j = j0; j < j1; ++j) nc += (modality[j] != 0) == (cand_mod != 0);
+    int tot;
+    const int cbase = block_exclusive_scan(nc, scan_buf, &tot);
+    {
+        int cr = cbase;
+        for (int j = j0; j < j1; ++j)
+            if ((modality[j] != 0) == (cand_mod != 0)) {
+                if (is_sink(p, j) && cr < n_cand) keys[cr] = 0u;
+                ++cr;
+            }
+    }
+    __syncthreads();
+
+    // ---- radix select of the slots-th largest key
+    uint32_t prefix = 0;
+    int kk = c.slots;
+    if (c.slots > 0) {
+        for (int shift = 24; shift >= 0; shift -= 8) {
+            hist[tid] = 0;   // kThreads == 256 bins
+            __syncthreads();
+            const uint32_t hi_mask = (shift == 24) ? 0u : (0xFFFFFFFFu << (shift + 8));
+            for (int i = tid; i < n_cand; i += kThreads) {
+                const uint32_t key = keys[i];
+                if ((key & hi_mask) == (prefix & hi_mask)) atomicAdd(&hist[(key >> shift) & 255], 1);
+            }
+            __syncthreads();
+            if (warp == 0) {
+                int cnt[8];
+                int sum = 0;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    cnt[e] = hist[255 - 8 * lane - e];
+                    sum += cnt[e];
+                }
+                int incl = sum;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const int y = __shfl_up_sync(~0u, incl, o);
+                    if (lane >= o) incl += y;
+                }
+                const int above = incl - sum;
+                if (above < kk && kk <= above + sum) {
+                    int a = above;
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        if (kk <= a + cnt[e]) {
+                            s_prefix = prefix | ((uint32_t)(255 - 8 * lane - e) << shift);
+                            s_kk = kk - a;
+                            break;
+                        }
+                        a += cnt[e];
+                    }
+                }
+            }
+            __syncthreads();
+            prefix = s_prefix;
+            kk = s_kk;
+        }
+    }
+    const bool none = c.slots == 0;
+    const uint32_t thr = prefix;
+    const int k_eq = none ? 0 : kk;
+
+    // ---- ordered emission
+    int neq = 0;
+    if (!none) {
+        int cr = cbase;
+        for (int j = j0; j < j1; ++j)
+            if ((modality[j] != 0) == (cand_mod != 0)) {
+                neq += (cr < n_cand && !is_sink(p, j) && keys[cr] == thr);
+                ++cr;
+            }
+    }
+    const int ebase = block_exclusive_scan(neq, scan_buf, &tot);
+    // kept(j): a sink, a text key when vision keys are ranked, or a ranked
+    // candidate above T, or one of the first k_eq equal to T
+    auto scan_kept = [&](auto&& emit) {
+        int cr = cbase, er = ebase;
+        for (int j = j0; j < j1; ++j) {
+            const bool isc = (modality[j] != 0) == (cand_mod != 0);
+            bool keep = is_sink(p, j) || (c.vision && modality[j] == 0);
+            if (isc) {
+                if (!keep && !none && cr < n_cand) {
+                    const uint32_t key = keys[cr];
+                    if (key > thr) {
+                        keep = true;
+                    } else if (key == thr) {
+                        keep = er < k_eq;
+                        ++er;
+                    }
+                }
+                ++cr;
+            }
+            if (keep) emit(j);
+        }
+    };
+    int nkeep = 0;
+    scan_kept([&](int) { ++nkeep; });
+    const int kbase = block_exclusive_scan(nkeep, scan_buf, &tot);
+    const long long off = s_off;
+    {
+        int r = kbase;
+        scan_kept([&](int j) {
+            if (r < len) {
+                idx[off + r] = j;
+                if (COMPACT) rows[r] = j;
+            }
+            ++r;
+        });
+    }
+    if (tid == 0 && tot != len) raise_status(status, TGVKV_STATUS_COUNT);
+    if (!COMPACT) return;
+
+    __syncthreads();
+    constexpr int RPI = 32 / VPR;
+    constexpr int UNROLL = 4;
+    const int n = min(len, tot);
+    const int sub = lane / VPR, vec = lane % VPR;
+    const size_t head = (size_t)lg * p.N;
+    for (int r0 = warp * RPI * UNROLL; r0 < n; r0 += (kThreads / 32) * RPI * UNROLL) {
+        uint4 kr[UNROLL], vr[UNROLL];
+#pragma unroll
+        for (int u = 0; u < UNROLL; ++u) {
+            const int r = r0 + u * RPI + sub;
+            if (r < n) {
+                const size_t src = (head + rows[r]) * VPR + vec;
+                kr[u] = __ldg(k + src);
+                vr[u] = __ldg(v + src);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < UNROLL; ++u) {
+            const int r = r0 + u * RPI + sub;
+            if (r < n) {
+                const size_t dst = (size_t)(off + r) * VPR + vec;
+                k_out[dst] = kr[u];
+                v_out[dst] = vr[u];
+            }
+        }
+    }
+}
+
+template <bool COMPACT, int VPR>
+cudaError_t launch_sel_general(const Problem& p, const float* scores, const float* text_scores,
+                               const int32_t* budgets, const uint8_t* modality, int64_t* offsets,
+                               int32_t* idx, const uint16_t* k, const uint16_t* v, uint16_t* k_out,
+                               uint16_t* v_out, uint32_t* status, cudaStream_t stream) {
+    auto kern = tpr_select_general_kernel<COMPACT, VPR>;
+    const size_t smem = select_general_smem(p, COMPACT);
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    kern<<<p.L * p.H_kv, kThreads, smem, stream>>>(
+        p, scores, text_scores, budgets, modality, offsets, idx, reinterpret_cast<const uint4*>(k),
+        reinterpret_cast<const uint4*>(v), reinterpret_cast<uint4*>(k_out),
+        reinterpret_cast<uint4*>(v_out), status);
+    return cudaGetLastError();
+}
+
+// The hot-path kernels cover the vision basis without sinks.
+inline bool general_select(const Problem& p) {
+    return p.basis == TGVKV_BASIS_ALL || p.keep_first > 0 || p.keep_last > 0;
+}
+
 // Warps per CTA of the warp-per-head kernel for p (0: use the CTA-per-head
 // kernel): only when there are many heads and eight heads' tables fit in
 // 64 KB, so that enough warps share an SM to keep the gather's loads in
@@ -454,22 +723,41 @@ cudaError_t launch_sel(const Problem& p, const float* scores, const int32_t* bud
 
 }  // namespace
 
-cudaError_t launch_select(const Problem& p, const float* scores, const int32_t* budgets,
-                          const uint8_t* modality, int64_t* offsets, int32_t* idx,
-                          uint32_t* status, cudaStream_t stream) {
+cudaError_t launch_select(const Problem& p, const float* scores, const float* text_scores,
+                          const int32_t* budgets, const uint8_t* modality, int64_t* offsets,
+                          int32_t* idx, uint32_t* status, cudaStream_t stream) {
+    if (general_select(p))
+        return launch_sel_general<false, 16>(p, scores, text_scores, budgets, modality, offsets,
+                                             idx, nullptr, nullptr, nullptr, nullptr, status,
+                                             stream);
     return launch_sel<false, 16>(p, scores, budgets, modality, offsets, idx, nullptr, nullptr, nullptr,
                                  nullptr, status, stream);
 }
 
 int select_compact_launches(const Problem& p) {
+    if (general_select(p)) return select_general_smem(p, true) > kFusedSmemLimit ? 2 : 1;
     return warp_select_warps(p) == 0 && select_smem(p, true) > kFusedSmemLimit ? 2 : 1;
 }
 
-cudaError_t launch_select_compact(const Problem& p, const float* scores, const int32_t* budgets,
-                                  const uint8_t* modality, int64_t* offsets, int32_t* idx,
-                                  const uint16_t* k, const uint16_t* v, uint16_t* k_out,
-                                  uint16_t* v_out, long long capacity_rows, uint32_t* status,
-                                  cudaStream_t stream) {
+cudaError_t launch_select_compact(const Problem& p, const float* scores, const float* text_scores,
+                                  const int32_t* budgets, const uint8_t* modality,
+                                  int64_t* offsets, int32_t* idx, const uint16_t* k,
+                                  const uint16_t* v, uint16_t* k_out, uint16_t* v_out,
+                                  long long capacity_rows, uint32_t* status, cudaStream_t stream) {
+    if (general_select(p)) {
+        if (select_general_smem(p, true) > kFusedSmemLimit) {
+            cudaError_t e = launch_select(p, scores, text_scores, budgets, modality, offsets, idx,
+                                          status, stream);
+            if (e != cudaSuccess) return e;
+            return launch_compact(p, k, v, offsets, idx, k_out, v_out, capacity_rows, status,
+                                  stream);
+        }
+        if (p.d == 64)
+            return launch_sel_general<true, 8>(p, scores, text_scores, budgets, modality, offsets,
+                                               idx, k, v, k_out, v_out, status, stream);
+        return launch_sel_general<true, 16>(p, scores, text_scores, budgets, modality, offsets, idx,
+                                            k, v, k_out, v_out, status, stream);
+    }
     if (const int nw = warp_select_warps(p)) {
         if (p.d == 64)
             return launch_sel_warp<8>(p, nw, scores, budgets, modality, offsets, idx, k, v, k_out,
@@ -478,7 +766,8 @@ cudaError_t launch_select_compact(const Problem& p, const float* scores, const i
                                    v_out, status, stream);
     }
     if (select_smem(p, true) > kFusedSmemLimit) {
-        cudaError_t e = launch_select(p, scores, budgets, modality, offsets, idx, status, stream);
+        cudaError_t e = launch_select(p, scores, nullptr, budgets, modality, offsets, idx, status,
+                                      stream);
         if (e != cudaSuccess) return e;
         return launch_compact(p, k, v, offsets, idx, k_out, v_out, capacity_rows, status, stream);
     }

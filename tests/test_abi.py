@@ -107,3 +107,37 @@ def test_evict_launch_count(lib):
     assert lib.tgvkv_evict_launches(ref(_desc(n_win=0))) == 2
     assert lib.tgvkv_evict_launches(ref(_desc(d=32))) == -1
     assert lib.tgvkv_evict_launches(None) == -1
+
+
+def test_all_basis_and_sink_arithmetic_matches_oracle(lib):
+    """The all-token basis shares out floor(r * N * L + 1/2) rows; sinks add at
+    most one row per sink to each (layer, head) set."""
+    ref = ctypes.byref
+    for wl in synth.WORKLOADS.values():
+        base = dict(L=wl.L, H_q=wl.H_q, H_kv=wl.H_kv, d=wl.d, N=wl.N, N_v=wl.N_v, n_win=wl.n_win,
+                    w_layer_stride=wl.n_win)
+        d_all = _desc(**base, budget_basis=1)
+        d_snk = _desc(**base, keep_first=4, keep_last=1)
+        for r in (0.0, 0.05, 0.2, 1.0):
+            b = oracle.all_budget_total(r, wl.N, wl.L)
+            assert lib.tgvkv_budget_total(ref(d_all), r) == b
+            assert lib.tgvkv_retained_rows(ref(d_all), r) == wl.H_kv * b
+            bv = oracle.vision_budget_total(r, wl.N_v, wl.L)
+            assert lib.tgvkv_budget_total(ref(d_snk), r) == bv
+            assert lib.tgvkv_retained_rows(ref(d_snk), r) == wl.H_kv * (wl.L * (wl.N_t + 5) + bv)
+    assert lib.tgvkv_budget_total(ref(_desc(budget_basis=2)), 0.1) == -1
+    assert lib.tgvkv_budget_total(ref(_desc(weight_mode=3)), 0.1) == -1
+    assert lib.tgvkv_budget_total(ref(_desc(keep_first=-1)), 0.1) == -1
+
+
+def test_evict_launch_count_with_text_pass(lib):
+    """Eq. 7 weights add the text-key score pass and the weights kernel; the
+    all-token basis adds the text-key pass (its Eq. 9 scores feed Eq. 10)."""
+    ref = ctypes.byref
+    for wl in synth.WORKLOADS.values():
+        base = dict(L=wl.L, H_q=wl.H_q, H_kv=wl.H_kv, d=wl.d, N=wl.N, N_v=wl.N_v, n_win=wl.n_win,
+                    w_layer_stride=wl.n_win)
+        assert lib.tgvkv_evict_launches(ref(_desc(**base, weight_mode=1))) == 4, wl.name
+        assert lib.tgvkv_evict_launches(ref(_desc(**base, budget_basis=1))) == 3, wl.name
+        assert lib.tgvkv_evict_launches(ref(_desc(**base, budget_basis=1, weight_mode=1))) == 4
+        assert lib.tgvkv_evict_launches(ref(_desc(**base, keep_first=4, keep_last=1))) == 2

@@ -1,0 +1,234 @@
+"""GPU parity of the widened path: Eq. 9 text scores, Eq. 7 derived weights,
+the all-token budget basis with both cases of Eq. 10, and sink tokens -- the
+CUDA path through the C ABI against the fp64 oracle.
+
+Tolerances: text scores and weights within 1e-3 relative (fp32 accumulation,
+as the vision scores).  Vision scores computed with the GPU's derived weights
+are compared with the oracle fed those same weights (1e-3); against the
+oracle's own Eq. 7 weights the bound is 2e-3, the weights' relative error
+adding to the attention's (the score is a positive combination of attention
+entries with those weights).  Budgets, retained sets and compacted rows are
+exact given the GPU's statistic and scores (integer decisions in the same
+fp32 values on both sides).
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2606_03075_gb300 import synth
+
+import _parity as P
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def api():
+    assert torch.cuda.is_available(), "the GPU tests need a CUDA device"
+    from paper_2606_03075_gb300 import build
+    build.build()
+    from paper_2606_03075_gb300 import api as _api
+    return _api
+
+
+def _video_like(frames, stamp, per_frame, head, tail):
+    s = [("text", head)]
+    for _ in range(frames):
+        s += [("text", stamp), ("vision", per_frame)]
+    return s + [("text", tail)]
+
+
+CASES = {
+    # several key tiles, a ragged tail, MHA with one row tile per head
+    "mha_single": synth.custom("mha_single", 2, 4, 4, 128,
+                               [("text", 13), ("vision", 300), ("text", 9), ("vision", 61),
+                                ("text", 90)], ratios=(0.1,)),
+    # two heads per row tile (<= 64 rows), d = 64
+    "mha_packed_d64": synth.custom("mha_packed_d64", 3, 4, 4, 64,
+                                   [("text", 20), ("vision", 180), ("text", 40)], ratios=(0.2,)),
+    # grouped-query heads, several row tiles per head, text interleaved
+    "gqa_pairs": synth.custom("gqa_pairs", 2, 14, 2, 128, _video_like(6, 5, 40, 9, 30),
+                              window="all_text", weights="dirichlet", ratios=(0.05,)),
+    # text longer than vision
+    "text_heavy": synth.custom("text_heavy", 2, 8, 2, 128,
+                               [("text", 150), ("vision", 64), ("text", 200)], window=120,
+                               ratios=(0.3,)),
+}
+
+
+def _oracle_text(wl, inp, layers=None):
+    return oracle.text_scores_and_weights(oracle.widen_bf16(inp["q"]), oracle.widen_bf16(inp["k"]),
+                                          inp["modality"], inp["text_pos"], 1.0 / math.sqrt(wl.d),
+                                          wl.H_kv, layers)
+
+
+def _run_text(api, wl, dev):
+    desc = api.desc_for_workload(wl)
+    ws = api.new_workspace(desc)
+    ts = torch.empty((wl.L, wl.H_kv, wl.N_t), dtype=torch.float32, device="cuda")
+    wt = torch.empty((wl.L, wl.n_win), dtype=torch.float32, device="cuda")
+    api.tgvkv_text_scores(desc, dev["q"], dev["k"], dev["modality"], dev["text_pos"], ts, wt, ws)
+    assert api.tgvkv_status(ws) == 0
+    return ts.cpu().numpy(), wt.cpu().numpy()
+
+
+@pytest.mark.parametrize("name", sorted(CASES))
+def test_text_scores_and_eq7_weights(api, name):
+    wl = CASES[name]
+    inp = synth.generate(wl, seed=1)
+    ts, wt = _run_text(api, wl, P.device_inputs(inp))
+    rts, rwt = _oracle_text(wl, inp)
+    P.assert_close(ts, rts, "text scores (Eq. 9)")
+    P.assert_close(wt, rwt, "weights (Eq. 7)")
+    assert np.allclose(wt.sum(axis=1), 1.0, rtol=1e-5)
+
+
+@pytest.mark.parametrize("name,layers", [("llava15", [0, 31]), ("qwen25", [5]), ("video", [27])])
+def test_text_scores_full_size_sampled(api, name, layers):
+    """Full-size shapes in the launch configuration tgvkv_evict uses, checked on
+    sampled layers (the oracle evaluates only those)."""
+    wl = synth.WORKLOADS[name]
+    inp = synth.generate(wl, seed=0)
+    ts, wt = _run_text(api, wl, P.device_inputs(inp))
+    rts, rwt = _oracle_text(wl, inp, layers)
+    P.assert_close(ts[layers], rts[layers], "text scores (Eq. 9)")
+    P.assert_close(wt[layers], rwt[layers], "weights (Eq. 7)")
+
+
+def _evict(api, wl, inp, ratio, **opts):
+    desc = api.desc_for_workload(wl, **opts)
+    dev = P.device_inputs(inp)
+    ws = api.new_workspace(desc)
+    out = api.alloc_outputs(desc, ratio)
+    w = None if opts.get("weights") == "eq7" else dev["w"]
+    api.tgvkv_evict(desc, dev["q"], dev["k"], dev["v"], dev["modality"], dev["text_pos"], w,
+                    ratio, out, ws)
+    status = api.tgvkv_status(ws)
+    n = int(out.offsets[-1].item())
+    assert n <= api.tgvkv_retained_rows(desc, ratio)
+    return dict(scores=out.scores.cpu().numpy(), stat=out.tvb_stat.cpu().numpy(),
+                budgets=out.budgets.cpu().numpy().astype(np.int64),
+                offsets=out.offsets.cpu().numpy(), idx=out.idx[:n].cpu().numpy().astype(np.int64),
+                k_out=out.k_out[:n].view(torch.int16).cpu().numpy(),
+                v_out=out.v_out[:n].view(torch.int16).cpu().numpy(), status=status, dev=dev,
+                desc=desc)
+
+
+@pytest.mark.parametrize("name", sorted(CASES))
+def test_evict_with_eq7_weights(api, name):
+    wl = CASES[name]
+    inp = synth.generate(wl, seed=2)
+    g = _evict(api, wl, inp, wl.ratios[0], weights="eq7")
+    assert g["status"] == 0
+    _, gw = _run_text(api, wl, g["dev"])
+    q, k = oracle.widen_bf16(inp["q"]), oracle.widen_bf16(inp["k"])
+    scale = 1.0 / math.sqrt(wl.d)
+    # the scores of the evict call, against the oracle fed the GPU's weights
+    s_gw, st = oracle.twr_scores_tvb_stat(q, k, inp["modality"], inp["text_pos"],
+                                          gw.astype(np.float64), scale, wl.H_kv)
+    P.assert_close(g["scores"], s_gw, "scores with the GPU's Eq. 7 weights")
+    P.assert_close(g["stat"], st, "tvb_stat")
+    # end to end against the oracle's own Eq. 7 weights
+    ref = oracle.evict(inp["q"], inp["k"], inp["v"], inp["modality"], inp["text_pos"], None,
+                       wl.ratios[0], wl.H_kv, weights="eq7")
+    P.assert_close(g["scores"], ref["scores"], "scores (Eq. 7 end to end)", rtol=2e-3)
+    # selection and compaction exact given the GPU's scores and budgets
+    assert g["budgets"].tolist() == oracle.tvb_budgets(g["stat"], oracle.vision_budget_total(
+        wl.ratios[0], wl.N_v, wl.L), wl.N_v)
+    P.check_selection_and_compaction(wl, inp, g, list(range(wl.L)))
+
+
+def _check_general(wl, inp, g, ratio, basis, keep):
+    """Budgets from the GPU statistic and the retained sets from the GPU scores,
+    exactly as the oracle decides them."""
+    if basis == "all":
+        total, cap = oracle.all_budget_total(ratio, wl.N, wl.L), wl.N
+    else:
+        total, cap = oracle.vision_budget_total(ratio, wl.N_v, wl.L), wl.N_v
+    assert g["budgets"].tolist() == oracle.tvb_budgets(g["stat"], total, cap)
+    ts = g.get("text_scores")
+    off, idx = oracle.tpr_select_general(g["scores"], ts, g["budgets"], inp["modality"], *keep,
+                                         vision_basis=basis == "vision")
+    np.testing.assert_array_equal(g["offsets"], off)
+    np.testing.assert_array_equal(g["idx"], idx)
+    ko, vo = oracle.compact(inp["k"], inp["v"], off, idx)
+    np.testing.assert_array_equal(g["k_out"], ko)
+    np.testing.assert_array_equal(g["v_out"], vo)
+
+
+@pytest.mark.parametrize("name", sorted(CASES))
+@pytest.mark.parametrize("ratio", [0.02, 0.3, 0.9])
+def test_evict_all_token_basis(api, name, ratio):
+    """Ratios that put layers in both cases of Eq. 10 (b_l <= N_t: text only;
+    b_l > N_t: all text plus vision)."""
+    wl = CASES[name]
+    inp = synth.generate(wl, seed=3)
+    g = _evict(api, wl, inp, ratio, basis="all")
+    assert g["status"] == 0
+    ts, _ = _run_text(api, wl, g["dev"])
+    g["text_scores"] = ts
+    ref = oracle.evict(inp["q"], inp["k"], inp["v"], inp["modality"], inp["text_pos"], inp["w"],
+                       ratio, wl.H_kv, basis="all")
+    P.assert_close(g["scores"], ref["scores"], "scores")
+    P.assert_close(ts, ref["text_scores"], "text scores")
+    _check_general(wl, inp, g, ratio, "all", (0, 0))
+    assert g["offsets"][-1] == wl.H_kv * oracle.all_budget_total(ratio, wl.N, wl.L)
+
+
+SINK_CASE = synth.custom("sinks", 3, 6, 2, 128,
+                         [("vision", 6), ("text", 11), ("vision", 200), ("text", 30),
+                          ("vision", 3)], window=30, ratios=(0.1,))
+
+
+@pytest.mark.parametrize("basis", ["vision", "all"])
+@pytest.mark.parametrize("keep", [(4, 1), (8, 5)])
+@pytest.mark.parametrize("ratio", [0.0, 0.05, 0.5])
+def test_evict_with_sinks(api, basis, keep, ratio):
+    """Sinks on vision and text tokens at both ends of the sequence."""
+    wl = SINK_CASE
+    inp = synth.generate(wl, seed=4)
+    g = _evict(api, wl, inp, ratio, basis=basis, keep_first=keep[0], keep_last=keep[1])
+    assert g["status"] == 0
+    if basis == "all":
+        g["text_scores"], _ = _run_text(api, wl, g["dev"])
+    _check_general(wl, inp, g, ratio, basis, keep)
+    sinks = oracle.sink_positions(wl.N, *keep)
+    H = wl.H_kv
+    for lg in range(wl.L * H):
+        assert set(sinks.tolist()) <= set(g["idx"][g["offsets"][lg]:g["offsets"][lg + 1]].tolist())
+
+
+def test_select_tpr_call_matches_evict(api):
+    """The separate calls (text scores, score, budget, select_tpr, compact)
+    give the fused call's result under the all-token basis with sinks."""
+    wl = CASES["gqa_pairs"]
+    inp = synth.generate(wl, seed=5)
+    ratio = 0.3
+    g = _evict(api, wl, inp, ratio, basis="all", keep_first=4, keep_last=1)
+    desc, dev = g["desc"], g["dev"]
+    ws = api.new_workspace(desc)
+    ts = torch.empty((wl.L, wl.H_kv, wl.N_t), dtype=torch.float32, device="cuda")
+    wt = torch.empty((wl.L, wl.n_win), dtype=torch.float32, device="cuda")
+    api.tgvkv_text_scores(desc, dev["q"], dev["k"], dev["modality"], dev["text_pos"], ts, wt, ws)
+    sc = torch.empty((wl.L, wl.H_kv, wl.N_v), dtype=torch.float32, device="cuda")
+    st = torch.empty(wl.L, dtype=torch.float32, device="cuda")
+    api.tgvkv_score(desc, dev["q"], dev["k"], dev["modality"], dev["text_pos"], dev["w"], sc, st, ws)
+    bud = torch.empty(wl.L, dtype=torch.int32, device="cuda")
+    api.tgvkv_budget(desc, st, ratio, bud, ws)
+    rows = api.tgvkv_retained_rows(desc, ratio)
+    off = torch.empty(wl.L * wl.H_kv + 1, dtype=torch.int64, device="cuda")
+    idx = torch.empty(rows, dtype=torch.int32, device="cuda")
+    api.tgvkv_select_tpr(desc, sc, ts, bud, dev["modality"], off, idx, ws)
+    n = int(off[-1].item())
+    ko = torch.empty((rows, wl.d), dtype=torch.bfloat16, device="cuda")
+    vo = torch.empty_like(ko)
+    api.tgvkv_compact(desc, dev["k"], dev["v"], off, idx, ko, vo, ws)
+    assert api.tgvkv_status(ws) == 0
+    np.testing.assert_array_equal(off.cpu().numpy(), g["offsets"])
+    np.testing.assert_array_equal(idx[:n].cpu().numpy(), g["idx"])
+    np.testing.assert_array_equal(ko[:n].view(torch.int16).cpu().numpy(), g["k_out"])
+    with pytest.raises(api.TgvkvError):
+        api.tgvkv_select(desc, sc, bud, dev["modality"], off, idx, ws)
