@@ -47,11 +47,15 @@ def parse():
     ap.add_argument("--impl", default="tgvkv", choices=["tgvkv", "reference"])
     ap.add_argument("--config", default="llava15", choices=sorted(synth.WORKLOADS))
     ap.add_argument("--ratio", type=float, default=None)
+    ap.add_argument("--layers", type=int, default=0,
+                    help="profiling: cut the workload to this many layers (0 = all)")
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="wall-clock target of the oracle CPU-baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-next-rows", action="store_true",
+                    help="skip timing the Eq. 7 / all-token basis / sink variants of the step")
     ap.add_argument("--record-traffic", metavar="CSV",
                     help="record the DRAM bytes of one kernel launch from `ncu -i REP --page raw "
                          "--csv` output into profiles/traffic.json (for --stage and --config)")
@@ -62,6 +66,16 @@ def parse():
 # --------------------------------------------------------------------------
 # workload description and algorithmic byte counts
 # --------------------------------------------------------------------------
+def workload_of(args):
+    """The named workload, cut to --layers layers when given (small profiling
+    cases of the same launch configuration)."""
+    wl = synth.WORKLOADS[args.config]
+    if args.layers:
+        import dataclasses
+        wl = dataclasses.replace(wl, L=args.layers)
+    return wl
+
+
 def workload_config(wl, ratio):
     return {"workload": f"{wl.name}: L={wl.L} H_q/H_kv={wl.H_q}/{wl.H_kv} d={wl.d} "
                         f"N={wl.N} (N_v={wl.N_v}, N_t={wl.N_t}) query rows={wl.n_win} "
@@ -286,12 +300,17 @@ def _oracle_units_worker(job):
     return time.perf_counter() - t
 
 
+_ARM_PARTS = {"0xd4f": "Arm Neoverse-V2", "0xd40": "Arm Neoverse-V1", "0xd0c": "Arm Neoverse-N1",
+              "0xd49": "Arm Neoverse-N2"}
+
+
 def cpu_model():
     try:
         for line in open("/proc/cpuinfo"):
             key = line.split(":")[0].strip().lower()
             if key in ("model name", "cpu part", "hardware"):
-                return line.split(":", 1)[1].strip()
+                val = line.split(":", 1)[1].strip()
+                return _ARM_PARTS.get(val.lower(), val)
     except OSError:
         pass
     import platform
@@ -303,7 +322,10 @@ def run_cpu_baseline(wl, ratio, seed, seconds):
     single-threaded process per core over (layer, KV head) units)."""
     import multiprocessing as mp
     cores = os.cpu_count() or 1
-    units = [(l, g) for l in range(wl.L) for g in range(wl.H_kv)]
+    all_units = [(l, g) for l in range(wl.L) for g in range(wl.H_kv)]
+    # the sample cycles over the workload's units when the whole workload takes
+    # less than the time asked for
+    units = [all_units[i % len(all_units)] for i in range(64 * len(all_units))]
     saved = {k: os.environ.get(k) for k in _ONE_THREAD}
     os.environ.update(_ONE_THREAD)
     try:
@@ -334,7 +356,8 @@ def run_cpu_baseline(wl, ratio, seed, seconds):
     return {"value": multi, "unit": UNIT, "cores": cores, "kind": "oracle",
             "single_thread_value": single, "cpu_model": cpu_model(),
             "sample": f"fp64 numpy oracle, BLAS one thread per process: {n} (layer, KV head) "
-                      f"units of {wl.name} single-threaded ({spent1:.1f} s), then {per_core} "
+                      f"units of {wl.name} (cycling over its {len(all_units)}) single-threaded "
+                      f"({spent1:.1f} s), then {per_core} "
                       f"units on each of {cores} cores in parallel processes ({wall:.1f} s wall); "
                       f"us/layer = time per unit x H_kv={wl.H_kv} (value: all cores)"}
 
@@ -345,7 +368,7 @@ def run_cpu_baseline(wl, ratio, seed, seconds):
 def run_reference(args, rank, world):
     if rank != 0:
         return 0
-    wl = synth.WORKLOADS[args.config]
+    wl = workload_of(args)
     ratio = args.ratio if args.ratio is not None else wl.ratios[0]
     units = [(l, g) for l in range(wl.L) for g in range(wl.H_kv)]
     cache = {}
@@ -406,7 +429,7 @@ def main():
     if world > 1:
         dist.init_process_group("nccl", device_id=dev)
 
-    wl = synth.WORKLOADS[args.config]
+    wl = workload_of(args)
     ratio = args.ratio if args.ratio is not None else wl.ratios[0]
     desc = api.desc_for_workload(wl)
     inp = synth.generate(wl, seed=args.seed + rank)
@@ -487,6 +510,47 @@ def main():
     barrier()
     stage_ms = {st: statistics.mean(sev[s][i].elapsed_time(sev[s][i + 1]) for s in range(args.steps))
                 for i, st in enumerate(stages)}
+
+    # ---- the widened path (Eq. 7 weights, all-token basis, sinks): the same
+    # evict call with the descriptor's options, inputs rotated as above
+    next_rows = {}
+    if not args.no_next_rows:
+        variants = {"eq7_weights": dict(weights="eq7"),
+                    "all_token_basis": dict(basis="all"),
+                    "sinks_4_1": dict(keep_first=4, keep_last=1),
+                    "eq7_all_sinks": dict(weights="eq7", basis="all", keep_first=4, keep_last=1)}
+        n_var = max(3, min(args.steps, 100))
+        for vname, opts in variants.items():
+            dv = api.desc_for_workload(wl, **opts)
+            wsv = api.new_workspace(dv, dev)
+            outv = api.alloc_outputs(dv, ratio, dev)
+
+            def evict_v(s):
+                x = sets[s % n_sets]
+                api.tgvkv_evict(dv, x["q"], x["k"], x["v"], x["modality"], x["text_pos"],
+                                None if opts.get("weights") == "eq7" else x["w"], ratio, outv,
+                                wsv, stream)
+
+            for s in range(3):
+                evict_v(s)
+            barrier()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            for s in range(n_var):
+                evict_v(3 + s)
+            b.record(stream)
+            barrier()
+            bits = api.tgvkv_status(wsv, stream)
+            if bits != 0:
+                raise RuntimeError(f"device status bits 0x{bits:x} set in the {vname} run")
+            bud = outv.budgets.cpu().numpy()
+            next_rows[vname] = {
+                "us_per_layer": a.elapsed_time(b) * 1e3 / (n_var * wl.L), "steps": n_var,
+                "launches_per_step": api.tgvkv_evict_launches(dv),
+                "rows_kept": int(outv.offsets[-1].item()),
+                "layers_text_only": int((bud <= wl.N_t).sum()) if opts.get("basis") == "all" else 0,
+                "options": opts}
+            del outv, wsv
 
     # ---- end to end through the public API with host buffers
     e2e = None
@@ -593,6 +657,7 @@ def main():
                          "peak_source": roof["peak_source"], "frac_nominal": roof["frac_nominal"]},
             "score_mufu": mufu,
             "stage_ms": stage_ms,
+            "next_rows": next_rows,
             "fused_tail_ms": statistics.mean(step_ms) - stage_ms["score"],
             "step_ms_median": statistics.median(step_ms),
             "wall_s_timed_region": t_wall,
