@@ -30,6 +30,8 @@
 //           [Q_0; Q_1] K_h^T, of which only head h's lanes are read (pass A),
 //           and K_h [Q_0; Q_1]^T, of which only head h's columns are read
 //           (pass B).  Every lane and every softmax thread does useful work.
+//           Two-head items fill whole rounds of the grid; the remaining heads
+//           are one-head items, so the last round spreads over more CTAs.
 //
 // Roles: warp 0 fetches items from a global counter (longest first) and issues
 // TMA loads -- an item's Q rows, then every K tile of both passes through a
@@ -132,8 +134,11 @@ __device__ __forceinline__ int q_box_row(const Item& it, int mode, int r, int g)
     return Item::pick(it.qy, r) + g * Item::pick(it.rpg, r);
 }
 
+// n_two: packed launches only -- items below n_two hold two heads, the rest
+// one head each (the last round of a launch, so that it spreads over more CTAs).
 template <int D>
-__device__ __forceinline__ Item item_info(const Problem& p, const PSmem<D>& s, int mode, int id) {
+__device__ __forceinline__ Item item_info(const Problem& p, const PSmem<D>& s, int mode, int id,
+                                          int n_two) {
     Item it;
     const int LH = p.L * p.H_kv;
     it.pidx = 0;
@@ -157,13 +162,15 @@ __device__ __forceinline__ Item item_info(const Problem& p, const PSmem<D>& s, i
         }
     } else {
         const bool packed = mode == MODE_PACKED;
+        const bool two = packed && id < n_two;
+        const int first = !packed ? id : (two ? 2 * id : n_two + id);
         it.nparts = 1;
 #pragma unroll
         for (int r = 0; r < 2; ++r) {
-            const int lh = packed ? 2 * id + r : id;
-            it.lh[r] = (r == 0 || (packed && lh < LH)) ? lh : -1;
+            const int lh = first + r;
+            it.lh[r] = (r == 0 || (two && lh < LH)) ? lh : -1;
             if (it.lh[r] >= 0 && r == 1) it.nparts = 2;
-            const int lhv = it.lh[r] >= 0 ? lh : id;
+            const int lhv = it.lh[r] >= 0 ? lh : first;
             it.l[r] = lhv / p.H_kv;
             it.qy[r] = (it.l[r] * p.H_q + (lhv % p.H_kv) * p.G) * p.n_win;
             it.rows[r] = p.R;
@@ -359,7 +366,7 @@ __device__ __forceinline__ void release_acc(uint64_t* bar, int lane) {
 template <int D, int MODE>
 __global__ void __launch_bounds__(NTHREADS, 1)
 score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
-                Problem p, int n_items, const uint8_t* __restrict__ modality,
+                Problem p, int n_items, int n_two, const uint8_t* __restrict__ modality,
                 const int32_t* __restrict__ text_pos, const float* __restrict__ w,
                 float* __restrict__ scores, float* __restrict__ tvb_stat,
                 float* __restrict__ score_part, float* __restrict__ stat_part,
@@ -507,7 +514,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
                 }
                 break;
             }
-            const Item itm = item_info(p, s, mode, id);
+            const Item itm = item_info(p, s, mode, id, n_two);
             // Q rows: pair items fill both slots (row tile r -> slot r); single
             // and packed items alternate slots.  Four boxes of 32 rows per slot,
             // box g landing in TMEM lanes 32g..32g+31.
@@ -594,7 +601,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
             const int id = s.item_q[slot];
             tc::mbar_arrive(&s.it_empty[slot]);
             if (id < 0) break;
-            const Item itm = item_info(p, s, mode, id);
+            const Item itm = item_info(p, s, mode, id, n_two);
             const int nslot = mode == MODE_PAIR ? itm.nparts : 1;
             const int qs0 = mode == MODE_PAIR ? 0 : (n & 1);
             for (int r = 0; r < nslot; ++r) {
@@ -697,7 +704,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
             tc::named_bar_sync(1, NSOFT);
             const int id = s.cur_item;
             if (id < 0) break;
-            const Item itm = item_info(p, s, mode, id);
+            const Item itm = item_info(p, s, mode, id, n_two);
 
             // ---- rows: lane 32q + i of row slot rs holds the part's row q*rpg + i
             // (packed: lanes 64h + 32q' + i hold head h's row q'*rpg + i)
@@ -1045,7 +1052,7 @@ int sm_count() {
 
 template <int D, int MODE>
 cudaError_t launch_mode(const CUtensorMap& mq, const CUtensorMap& mk, const Problem& p, int n_items,
-                        const uint8_t* modality, const int32_t* text_pos, const float* w,
+                        int n_two, const uint8_t* modality, const int32_t* text_pos, const float* w,
                         float* scores, float* tvb_stat, char* ws, const WsLayout& lay,
                         long long budget_total, int32_t* budgets, cudaStream_t stream) {
     static_assert(sizeof(PSmem<D>) + 1024 <= 227 * 1024, "shared memory of one CTA");
@@ -1060,7 +1067,7 @@ cudaError_t launch_mode(const CUtensorMap& mq, const CUtensorMap& mk, const Prob
     if (sms <= 0) return cudaErrorInvalidDevice;
     const int grid = n_items < sms ? n_items : sms;
     score_tc_kernel<D, MODE><<<grid, NTHREADS, smem, stream>>>(
-        mq, mk, p, n_items, modality, text_pos, w, scores, tvb_stat,
+        mq, mk, p, n_items, n_two, modality, text_pos, w, scores, tvb_stat,
         reinterpret_cast<float*>(ws + lay.score_part), reinterpret_cast<float*>(ws + lay.stat_part),
         reinterpret_cast<float*>(ws + lay.stat_head), reinterpret_cast<uint32_t*>(ws + lay.tickets),
         reinterpret_cast<uint32_t*>(ws + lay.status), budget_total, budgets);
@@ -1080,12 +1087,20 @@ cudaError_t launch_tc(const Problem& p, const uint16_t* q, const uint16_t* k,
     // heads of at most 64 rows each packed into one row tile
     const int LH = p.L * p.H_kv;
     if (p.T >= 2)
-        return launch_mode<D, MODE_PAIR>(mq, mk, p, LH * score_pairs(p), modality, text_pos, w,
+        return launch_mode<D, MODE_PAIR>(mq, mk, p, LH * score_pairs(p), 0, modality, text_pos, w,
                                          scores, tvb_stat, ws, lay, budget_total, budgets, stream);
-    if (2 * p.R <= BM)
-        return launch_mode<D, MODE_PACKED>(mq, mk, p, (LH + 1) / 2, modality, text_pos, w, scores,
+    if (2 * p.R <= BM) {
+        // Two heads per item in whole rounds of the grid, one head per item for
+        // the rest: the last round then spreads over up to twice as many CTAs
+        // (1024 heads on 152 SMs: 3 rounds of two-head items, 112 one-head items).
+        const int sms = sm_count();
+        if (sms <= 0) return cudaErrorInvalidDevice;
+        const int n_two = LH / 2 >= sms ? sms * ((LH / 2) / sms) : LH / 2;
+        const int n_items = n_two + (LH - 2 * n_two);
+        return launch_mode<D, MODE_PACKED>(mq, mk, p, n_items, n_two, modality, text_pos, w, scores,
                                            tvb_stat, ws, lay, budget_total, budgets, stream);
-    return launch_mode<D, MODE_SINGLE>(mq, mk, p, LH, modality, text_pos, w, scores, tvb_stat, ws,
+    }
+    return launch_mode<D, MODE_SINGLE>(mq, mk, p, LH, 0, modality, text_pos, w, scores, tvb_stat, ws,
                                        lay, budget_total, budgets, stream);
 }
 

@@ -178,7 +178,11 @@ __device__ __forceinline__ void mma_commit(uint64_t* bar) {
         : "memory");
 }
 
+// bar.sync is the warp-aligned form: every lane of a warp must execute it
+// together, so the warp is reconverged first (callers may have diverged on a
+// single-lane branch just before).
 __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
+    __syncwarp();
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
