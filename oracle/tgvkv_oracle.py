@@ -48,6 +48,11 @@ Beyond that hot path (same file, same conventions):
    "Implementation Details") are always kept and count against the part of the
    budget of their own modality.
 
+12. Decode over the compacted cache (the consumer of the step, Section 3.1
+   "Decode Phase"): a new token's query of head h attends to the retained
+   rows of its KV head g = h // G, ``o = softmax(scale * q K_I^T) V_I``; a head
+   with no retained row gives 0.
+
 Floating point: inputs are bf16 bit patterns widened exactly to float64; all
 arithmetic is float64.  The paper states no precision.
 
@@ -330,6 +335,34 @@ def compact(k_bits: np.ndarray, v_bits: np.ndarray, offsets, idx):
 def compacted_kv_bytes(offsets, head_dim: int, elem_bytes: int = 2) -> int:
     """Bytes of the compacted cache: K and V rows of every retained position."""
     return 2 * int(offsets[-1]) * head_dim * elem_bytes
+
+
+# --------------------------------------------------------------------------
+# Decode over the compacted cache
+# --------------------------------------------------------------------------
+def decode_attention(q: np.ndarray, k_rows: np.ndarray, v_rows: np.ndarray, offsets,
+                     n_kv_heads: int, scale: float) -> np.ndarray:
+    """One decode step of every layer over the compacted cache.
+
+    q:       [L, H_q, d] float64 queries of the new token.
+    k_rows, v_rows: [rows, d] float64 retained keys / values (CSR over (l, g)).
+    offsets: [L*H_kv + 1] CSR offsets.
+    Returns o [L, H_q, d]: o[l, h] = sum_r softmax_r(scale * <q[l,h], k_r>) v_r over
+    the rows r of set (l, h // G); zero for an empty set.
+    """
+    n_layers, n_q_heads, d = q.shape
+    group = n_q_heads // n_kv_heads
+    out = np.zeros((n_layers, n_q_heads, d))
+    for l in range(n_layers):
+        for h in range(n_q_heads):
+            lg = l * n_kv_heads + h // group
+            lo, hi = int(offsets[lg]), int(offsets[lg + 1])
+            if hi == lo:
+                continue
+            logits = scale * (k_rows[lo:hi] @ q[l, h])
+            e = np.exp(logits - logits.max())
+            out[l, h] = (e / e.sum()) @ v_rows[lo:hi]
+    return out
 
 
 # --------------------------------------------------------------------------

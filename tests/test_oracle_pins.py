@@ -575,3 +575,55 @@ def test_evict_eq7_and_all_basis_tiny():
         for l in range(L):
             for g in range(H_kv):
                 assert ra["offsets"][l * H_kv + g + 1] - ra["offsets"][l * H_kv + g] == ra["budgets"][l]
+
+
+# ---------------------------------------------------------------- decode over the compacted cache
+def _identity_csr(L, H_kv, n):
+    return np.arange(L * H_kv + 1, dtype=np.int64) * n
+
+
+def test_decode_full_cache_equals_causal_attention_row():
+    """With every row kept, decode equals the Eq. 2 attention row of a query
+    that sees all N keys, times V (the prefill definition, written separately)."""
+    rng = np.random.default_rng(50)
+    L, H_q, H_kv, d, n = 2, 6, 2, 8, 13
+    q = rng.standard_normal((L, H_q, d))
+    k = rng.standard_normal((L, H_kv, n, d))
+    v = rng.standard_normal((L, H_kv, n, d))
+    o = oracle.decode_attention(q, k.reshape(-1, d), v.reshape(-1, d), _identity_csr(L, H_kv, n),
+                                H_kv, 0.37)
+    for l in range(L):
+        for h in range(H_q):
+            a = oracle.causal_text_attention(q[l, h][None], k[l, h // 3], np.array([n - 1]), 0.37)
+            assert np.allclose(o[l, h], (a @ v[l, h // 3])[0], rtol=1e-12, atol=1e-14)
+
+
+def test_decode_uniform_and_saturated_and_empty():
+    rng = np.random.default_rng(51)
+    d, n = 6, 9
+    k = rng.standard_normal((n, d))
+    v = rng.standard_normal((n, d))
+    off = np.array([0, n, n], np.int64)          # layer 0 head 0 has n rows, head 1 none
+    q = np.zeros((1, 2, d))
+    o = oracle.decode_attention(q, k, v, off, 2, 1.0)
+    assert np.allclose(o[0, 0], v.mean(axis=0), rtol=1e-13)
+    assert np.array_equal(o[0, 1], np.zeros(d))
+    q[0, 0] = 80.0 * k[4] / np.linalg.norm(k[4]) ** 2 * 1.0
+    k2 = k.copy()
+    k2[4] *= 3.0
+    o = oracle.decode_attention(q, k2, v, off, 2, 1.0)
+    assert np.allclose(o[0, 0], v[4], atol=1e-9)
+
+
+def test_decode_row_order_does_not_matter():
+    rng = np.random.default_rng(52)
+    L, H_q, H_kv, d = 2, 4, 2, 5
+    lens = [3, 7, 1, 4]
+    off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    k = rng.standard_normal((off[-1], d))
+    v = rng.standard_normal((off[-1], d))
+    q = rng.standard_normal((L, H_q, d))
+    o = oracle.decode_attention(q, k, v, off, H_kv, 0.8)
+    perm = np.concatenate([off[i] + rng.permutation(lens[i]) for i in range(len(lens))])
+    o2 = oracle.decode_attention(q, k[perm], v[perm], off, H_kv, 0.8)
+    assert np.allclose(o, o2, rtol=1e-12, atol=1e-14)
