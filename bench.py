@@ -552,6 +552,57 @@ def main():
                 "options": opts}
             del outv, wsv
 
+    # ---- decode over the compacted cache vs over the full cache: the consumer
+    # of the step (one new token per layer), copies rotated past L2
+    decode = None
+    if not args.no_next_rows:
+        evict(0)
+        barrier()
+        n_rows = int(out.offsets[-1].item())
+        comp_bytes = 2 * n_rows * wl.d * 2
+        n_cp = max(2, math.ceil(2 * L2_BYTES / max(comp_bytes, 1)) + 1)
+        comp = [(out.k_out[:n_rows].clone(), out.v_out[:n_rows].clone()) for _ in range(n_cp)]
+        offs = out.offsets.clone()
+        full_off = torch.arange(wl.L * wl.H_kv + 1, dtype=torch.int64, device=dev) * wl.N
+        qdec = torch.from_numpy(synth.to_bf16_bits(
+            np.random.default_rng(args.seed + 11).standard_normal((wl.L, wl.H_q, wl.d))
+            .astype(np.float32))).to(dev).view(torch.bfloat16)
+        odec = torch.empty((wl.L, wl.H_q, wl.d), dtype=torch.float32, device=dev)
+        n_dec = max(3, min(args.steps, 200))
+
+        def time_decode(pick):
+            for s in range(3):
+                kk, vv, oo = pick(s)
+                api.tgvkv_decode(desc, qdec, kk, vv, oo, odec, ws, stream)
+            barrier()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            for s in range(n_dec):
+                kk, vv, oo = pick(3 + s)
+                api.tgvkv_decode(desc, qdec, kk, vv, oo, odec, ws, stream)
+            b.record(stream)
+            barrier()
+            return a.elapsed_time(b) * 1e3 / n_dec
+
+        t_comp = time_decode(lambda s: (comp[s % n_cp][0], comp[s % n_cp][1], offs))
+        t_full = time_decode(lambda s: (sets[s % n_sets]["k"], sets[s % n_sets]["v"], full_off))
+        bits = api.tgvkv_status(ws, stream)
+        if bits != 0:
+            raise RuntimeError(f"device status bits 0x{bits:x} set in the decode runs")
+        full_bytes = 2 * wl.L * wl.H_kv * wl.N * wl.d * 2
+        decode = {"what": "one decode step of every layer (one new token), attention over the "
+                          "cached K/V of each KV head's query heads",
+                  "compacted_us_per_token": t_comp, "full_us_per_token": t_full,
+                  "speedup": t_full / t_comp, "rows_compacted": n_rows,
+                  "rows_full": wl.L * wl.H_kv * wl.N,
+                  "compacted_gbs": comp_bytes / (t_comp * 1e-6) / 1e9,
+                  "full_gbs": full_bytes / (t_full * 1e-6) / 1e9,
+                  "launches": api.tgvkv_decode_launches(desc), "steps": n_dec}
+        pk = float(measured_peaks()[0]["hbm_gbs"])
+        decode["compacted_frac"] = decode["compacted_gbs"] / pk
+        decode["full_frac"] = decode["full_gbs"] / pk
+        del comp
+
     # ---- end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
@@ -658,6 +709,7 @@ def main():
             "score_mufu": mufu,
             "stage_ms": stage_ms,
             "next_rows": next_rows,
+            "decode": decode,
             "fused_tail_ms": statistics.mean(step_ms) - stage_ms["score"],
             "step_ms_median": statistics.median(step_ms),
             "wall_s_timed_region": t_wall,

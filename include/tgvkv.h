@@ -224,6 +224,25 @@ int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
  * budget kernel in place of the score kernel.  Returns -1 on bad arguments. */
 int tgvkv_evict_launches(const tgvkv_desc* desc);
 
+/* Decode over the compacted cache (the consumer of the eviction step; the
+ * decode phase of Section 3.1).  For one new token per layer, query head h of
+ * layer l attends to the rows of set (l, g = h / G) of a CSR cache:
+ *   out[l][h][:] = sum_r softmax_r(softmax_scale * <q[l][h], k_rows[r]>) v_rows[r]
+ * over r in [offsets[l*H_kv+g], offsets[l*H_kv+g+1]); an empty set gives 0.
+ * q: bf16 [L][H_q][d]; k_rows, v_rows: bf16 [rows][d] (k_out / v_out of
+ * tgvkv_evict, or the full cache [L][H_kv][N][d] with offsets[i] = i * N);
+ * offsets: int64 [L*H_kv + 1]; out: fp32 [L][H_q][d] (output).  bf16 products,
+ * fp32 accumulation and softmax.  The workspace holds the row-split partials
+ * (tgvkv_workspace_size covers them). */
+int tgvkv_decode(const tgvkv_desc* desc, const uint16_t* q, const uint16_t* k_rows,
+                 const uint16_t* v_rows, const int64_t* offsets, float* out,
+                 void* workspace, void* stream);
+
+/* Kernels one tgvkv_decode call launches (1, or 2 when few KV heads make it
+ * split each set's rows over several CTAs and merge them).  -1 on bad
+ * arguments. */
+int tgvkv_decode_launches(const tgvkv_desc* desc);
+
 /* Zero `workspace` (asynchronously on `stream`).  Needed once after the
  * workspace is allocated: the calls leave their completion counters at zero
  * for the next call.  Zero it again after a call whose tgvkv_status reported

@@ -52,6 +52,9 @@ SIGNATURES = {
     "tgvkv_workspace_init": (c_int, [_P, c_void_p, c_void_p]),
     "tgvkv_status": (c_int, [c_void_p, c_void_p]),
     "tgvkv_evict_launches": (c_int, [_P]),
+    "tgvkv_decode": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                             c_void_p]),
+    "tgvkv_decode_launches": (c_int, [_P]),
     "tgvkv_last_error": (c_char_p, []),
     "tgvkv_score_noalloc": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                     c_void_p, c_void_p, c_void_p]),

@@ -257,6 +257,24 @@ def tgvkv_status(ws: torch.Tensor, stream=None) -> int:
     return rc
 
 
+def tgvkv_decode(desc, q, k_rows, v_rows, offsets, out, ws, stream=None):
+    """One decode step of every layer over a CSR cache (see include/tgvkv.h)."""
+    L, Hq, Hkv, d = desc.L, desc.H_q, desc.H_kv, desc.d
+    _check(_lib.load().tgvkv_decode(
+        ctypes.byref(desc),
+        _ptr(q, _BF16_LIKE, L * Hq * d, "q"),
+        _ptr(k_rows, _BF16_LIKE, 0, "k_rows"),
+        _ptr(v_rows, _BF16_LIKE, 0, "v_rows"),
+        _ptr(offsets, (torch.int64,), L * Hkv + 1, "offsets"),
+        _ptr(out, (torch.float32,), L * Hq * d, "out"),
+        _ptr(ws, (torch.uint8,), tgvkv_workspace_size(desc), "workspace"),
+        _stream(stream)), "tgvkv_decode")
+
+
+def tgvkv_decode_launches(desc: Desc) -> int:
+    return int(_lib.load().tgvkv_decode_launches(ctypes.byref(desc)))
+
+
 def tgvkv_evict_launches(desc: Desc) -> int:
     """Kernels one tgvkv_evict call launches for this problem."""
     n = _lib.load().tgvkv_evict_launches(ctypes.byref(desc))

@@ -52,6 +52,9 @@ WsLayout layout_of(const Problem& p) {
     const size_t keyset = (size_t)(p.N_v > p.N_t ? p.N_v : p.N_t);
     if (p.T > 1) o += round_up(sizeof(float) * (size_t)p.L * p.H_kv * p.T * keyset);
     w.stat_text = o;   o += round_up(sizeof(float) * (size_t)p.L);
+    w.decode_part = o;
+    if (decode_splits(p) > 1)
+        o += round_up(sizeof(float) * (size_t)p.L * p.H_q * decode_splits(p) * (p.d + 2));
     w.text_scores = w.weights = 0;
     if (needs_text_pass(p)) {
         w.text_scores = o; o += round_up(sizeof(float) * (size_t)p.L * p.H_kv * (p.N_t > 0 ? p.N_t : 1));
@@ -396,6 +399,31 @@ int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
                               v_out, retained_rows(p, ratio), status, st);
     if (e != cudaSuccess) return cuda_fail(e, "select/compact launch");
     return ok();
+}
+
+int tgvkv_decode(const tgvkv_desc* desc, const uint16_t* q, const uint16_t* k_rows,
+                 const uint16_t* v_rows, const int64_t* offsets, float* out, void* workspace,
+                 void* stream) {
+    Problem p{};
+    int rc = make_problem(desc, &p);
+    if (rc) return rc;
+    REQUIRE_PTR(q, "q", false);
+    REQUIRE_PTR(k_rows, "k_rows", true);
+    REQUIRE_PTR(v_rows, "v_rows", true);
+    REQUIRE_PTR(offsets, "offsets", false);
+    REQUIRE_PTR(out, "out", false);
+    REQUIRE_PTR(workspace, "workspace", true);
+    const WsLayout lay = layout_of(p);
+    cudaError_t e = launch_decode(p, q, k_rows, v_rows, offsets, out,
+                                  reinterpret_cast<float*>(static_cast<char*>(workspace) + lay.decode_part),
+                                  static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ok() : cuda_fail(e, "decode launch");
+}
+
+int tgvkv_decode_launches(const tgvkv_desc* desc) {
+    Problem p{};
+    if (make_problem(desc, &p) != TGVKV_OK) return -1;
+    return decode_launches(p);
 }
 
 int tgvkv_evict_launches(const tgvkv_desc* desc) {

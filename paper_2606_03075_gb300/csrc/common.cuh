@@ -24,6 +24,17 @@ struct Problem {
     int keys_text;
 };
 
+// Row splits of the decode kernel: enough CTAs for two per SM on the 152 SMs
+// of a GB300 when there are few KV heads, at most one split per 128 positions.
+__host__ __device__ inline int decode_splits(const Problem& p) {
+    const int ctas = p.L * p.H_kv * ((p.G + 7) / 8);
+    int s = (2 * 152 + ctas - 1) / ctas;
+    const int most = (p.N + 127) / 128;
+    if (s > most) s = most;
+    if (s > 16) s = 16;
+    return s < 1 ? 1 : s;
+}
+
 // Sinks among the positions 0..N-1: the first keep_first and the last keep_last.
 __host__ __device__ inline bool is_sink(const Problem& p, int j) {
     return j < p.keep_first || j >= p.N - p.keep_last;
@@ -40,6 +51,7 @@ struct WsLayout {
     size_t text_scores; // float [L*H_kv*N_t]: Eq. 9 scores
     size_t weights;     // float [L*n_win]: Eq. 7 weights
     size_t stat_text;   // float [L]: the text-key pass's (unused) statistic
+    size_t decode_part; // float [L*H_q*S*(d+2)]: decode row-split partials (S > 1)
     size_t total;
 };
 

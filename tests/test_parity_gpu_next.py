@@ -232,3 +232,98 @@ def test_select_tpr_call_matches_evict(api):
     np.testing.assert_array_equal(ko[:n].view(torch.int16).cpu().numpy(), g["k_out"])
     with pytest.raises(api.TgvkvError):
         api.tgvkv_select(desc, sc, bud, dev["modality"], off, idx, ws)
+
+
+# ---------------------------------------------------------------- decode over the compacted cache
+def _decode_q(wl, seed):
+    rng = np.random.default_rng(seed)
+    return synth.to_bf16_bits(rng.standard_normal((wl.L, wl.H_q, wl.d)).astype(np.float32))
+
+
+def _run_decode(api, desc, q_bits, k_rows, v_rows, offsets):
+    ws = api.new_workspace(desc)
+    out = torch.empty((desc.L, desc.H_q, desc.d), dtype=torch.float32, device="cuda")
+    qd = torch.from_numpy(np.ascontiguousarray(q_bits)).cuda().view(torch.bfloat16)
+    api.tgvkv_decode(desc, qd, k_rows, v_rows, offsets, out, ws)
+    assert api.tgvkv_status(ws) == 0
+    return out.cpu().numpy()
+
+
+# A decode output is a convex combination of value rows: an entry that nearly
+# cancels (|o| far below its terms) carries the fp32 accumulation error of the
+# terms (~n * 6e-8 of them), so the absolute floor is 1e-5 of the head's largest
+# output rather than the scores' 1e-6.
+DEC_FLOOR = 1e-5
+
+
+def _oracle_decode(wl, q_bits, k_bits, v_bits, offsets):
+    return oracle.decode_attention(oracle.widen_bf16(q_bits), oracle.widen_bf16(k_bits),
+                                   oracle.widen_bf16(v_bits), offsets, wl.H_kv,
+                                   1.0 / math.sqrt(wl.d))
+
+
+DECODE_CASES = dict(CASES, tiny=synth.WORKLOADS["tiny"],
+                    wide_group=synth.custom("wide_group", 1, 32, 1, 128,
+                                            [("text", 3), ("vision", 90), ("text", 9)],
+                                            ratios=(0.5,)))
+
+
+@pytest.mark.parametrize("name", sorted(DECODE_CASES))
+def test_decode_over_compacted_cache(api, name):
+    """A decode step over the cache tgvkv_evict compacted, against the oracle on
+    the same retained rows (G > 8 takes several head batches per KV head)."""
+    wl = DECODE_CASES[name]
+    inp = synth.generate(wl, seed=6)
+    desc = api.desc_for_workload(wl)
+    dev = P.device_inputs(inp)
+    ws = api.new_workspace(desc)
+    ratio = wl.ratios[0]
+    out = api.alloc_outputs(desc, ratio)
+    api.tgvkv_evict(desc, dev["q"], dev["k"], dev["v"], dev["modality"], dev["text_pos"], dev["w"],
+                    ratio, out, ws)
+    assert api.tgvkv_status(ws) == 0
+    n = int(out.offsets[-1].item())
+    qb = _decode_q(wl, 7)
+    o = _run_decode(api, desc, qb, out.k_out, out.v_out, out.offsets)
+    ref = _oracle_decode(wl, qb, out.k_out[:n].view(torch.int16).cpu().numpy(),
+                         out.v_out[:n].view(torch.int16).cpu().numpy(), out.offsets.cpu().numpy())
+    P.assert_close(o, ref, "decode over the compacted cache", floor=DEC_FLOOR)
+
+
+@pytest.mark.parametrize("name", ["llava15", "qwen25"])
+def test_decode_full_size(api, name):
+    """Full-size caches: the compacted cache of tgvkv_evict and the full cache
+    (identity offsets), every layer and head against the oracle; qwen25 has few
+    KV heads, so its rows are split over several CTAs and merged."""
+    wl = synth.WORKLOADS[name]
+    inp = synth.generate(wl, seed=0)
+    desc = api.desc_for_workload(wl)
+    dev = P.device_inputs(inp)
+    ws = api.new_workspace(desc)
+    ratio = wl.ratios[0]
+    out = api.alloc_outputs(desc, ratio)
+    api.tgvkv_evict(desc, dev["q"], dev["k"], dev["v"], dev["modality"], dev["text_pos"], dev["w"],
+                    ratio, out, ws)
+    assert api.tgvkv_status(ws) == 0
+    qb = _decode_q(wl, 8)
+    n = int(out.offsets[-1].item())
+    o = _run_decode(api, desc, qb, out.k_out, out.v_out, out.offsets)
+    ref = _oracle_decode(wl, qb, out.k_out[:n].view(torch.int16).cpu().numpy(),
+                         out.v_out[:n].view(torch.int16).cpu().numpy(), out.offsets.cpu().numpy())
+    P.assert_close(o, ref, "decode, compacted cache", floor=DEC_FLOOR)
+    full_off = torch.arange(wl.L * wl.H_kv + 1, dtype=torch.int64, device="cuda") * wl.N
+    of = _run_decode(api, desc, qb, dev["k"], dev["v"], full_off)
+    reff = _oracle_decode(wl, qb, inp["k"].reshape(-1, wl.d), inp["v"].reshape(-1, wl.d),
+                          full_off.cpu().numpy())
+    P.assert_close(of, reff, "decode, full cache", floor=DEC_FLOOR)
+
+
+def test_decode_empty_sets_give_zero(api):
+    """No text token and a zero budget: every set is empty and the output is 0."""
+    wl = synth.custom("all_vision", 2, 4, 2, 64, [("vision", 70)], window="all_text",
+                      ratios=(0.0,))
+    desc = api.desc_for_workload(wl)
+    offsets = torch.zeros(wl.L * wl.H_kv + 1, dtype=torch.int64, device="cuda")
+    rows = torch.zeros((1, wl.d), dtype=torch.bfloat16, device="cuda")
+    o = _run_decode(api, desc, _decode_q(wl, 9), rows, rows, offsets)
+    assert np.array_equal(o, np.zeros_like(o))
