@@ -48,7 +48,11 @@ Beyond that hot path (same file, same conventions):
    "Implementation Details") are always kept and count against the part of the
    budget of their own modality.
 
-12. Decode over the compacted cache (the consumer of the step, Section 3.1
+12. Other layer-budget statistics (Table 1a, Eq. 5 with x in {VV, TT}):
+   ``S^TT_l = sum_{h,i} sum_{j in T} A_ij`` over the query rows; VV is the TV
+   statistic of item 3 computed with the vision tokens' queries as the rows;
+   uniform budgeting splits an all-zero statistic.
+13. Decode over the compacted cache (the consumer of the step, Section 3.1
    "Decode Phase"): a new token's query of head h attends to the retained
    rows of its KV head g = h // G, ``o = softmax(scale * q K_I^T) V_I``; a head
    with no retained row gives 0.
@@ -169,6 +173,21 @@ def text_scores_and_weights(q: np.ndarray, k: np.ndarray, modality: np.ndarray,
         w = w_sum / n_q_heads / rows_at_or_after
         weights[l] = w / w.sum()
     return t_scores, weights
+
+
+def tt_statistic(q: np.ndarray, k: np.ndarray, modality: np.ndarray, text_pos: np.ndarray,
+                 scale: float, n_kv_heads: int) -> np.ndarray:
+    """Eq. 5 with x = TT: per layer, the attention mass of the query rows on the
+    text keys, summed over every query head."""
+    n_layers, n_q_heads = q.shape[0], q.shape[1]
+    group = n_q_heads // n_kv_heads
+    text = np.flatnonzero(np.asarray(modality) == 0)
+    stat = np.zeros(n_layers)
+    for l in range(n_layers):
+        for h in range(n_q_heads):
+            a = causal_text_attention(q[l, h], k[l, h // group], text_pos, scale)
+            stat[l] += a[:, text].sum()
+    return stat
 
 
 # --------------------------------------------------------------------------
@@ -370,13 +389,16 @@ def decode_attention(q: np.ndarray, k_rows: np.ndarray, v_rows: np.ndarray, offs
 # --------------------------------------------------------------------------
 def evict(q_bits, k_bits, v_bits, modality, text_pos, w, ratio: float,
           n_kv_heads: int, scale: float | None = None, weights: str = "given",
-          basis: str = "vision", keep_first: int = 0, keep_last: int = 0):
+          basis: str = "vision", keep_first: int = 0, keep_last: int = 0,
+          budget_stat: str = "tv"):
     """Score, budget, select and compact, all in float64 on the host.
 
     weights: "given" uses ``w``; "eq7" derives w~ by Eq. 7 (``w`` is ignored).
     basis:   "vision" -- r counts vision KV and every text KV is kept (case
              b_l > N_t of Eq. 10 throughout); "all" -- r counts every KV and
              Eq. 10 applies per layer with the text scores of Eq. 9.
+    budget_stat: the statistic the layer budgets follow: "tv" (the method),
+             "tt" or "uniform" (Table 1a); the returned "stat" is the one split.
     """
     q = widen_bf16(q_bits)
     k = widen_bf16(k_bits)
@@ -394,6 +416,10 @@ def evict(q_bits, k_bits, v_bits, modality, text_pos, w, ratio: float,
             w = w_eq7
     w = np.asarray(w, dtype=np.float64)
     scores, stat = twr_scores_tvb_stat(q, k, modality, text_pos, w, scale, n_kv_heads)
+    if budget_stat == "tt":
+        stat = tt_statistic(q, k, modality, text_pos, scale, n_kv_heads)
+    elif budget_stat == "uniform":
+        stat = np.zeros(n_layers)
     if basis == "vision":
         total = vision_budget_total(ratio, n_vision, n_layers)
         budgets = tvb_budgets(stat, total, n_vision)

@@ -627,3 +627,51 @@ def test_decode_row_order_does_not_matter():
     perm = np.concatenate([off[i] + rng.permutation(lens[i]) for i in range(len(lens))])
     o2 = oracle.decode_attention(q, k[perm], v[perm], off, H_kv, 0.8)
     assert np.allclose(o, o2, rtol=1e-12, atol=1e-14)
+
+
+# ---------------------------------------------------------------- layer-budget statistics (Table 1a)
+def test_tt_statistic_ties_to_text_scores_and_tv():
+    """Eq. 5 with x = TT: the text-text mass equals G times the Eq. 9 text scores
+    summed, and with the TV mass fills every row (H_q * n_win per layer)."""
+    q, k, modality, pos, w = _rand_case(L=3, H_q=6, H_kv=2, d=7, seed=60)
+    tt = oracle.tt_statistic(q, k, modality, pos, 0.6, 2)
+    ts, _ = oracle.text_scores_and_weights(q, k, modality, pos, 0.6, 2)
+    _, tv = oracle.twr_scores_tvb_stat(q, k, modality, pos, w, 0.6, 2)
+    assert np.allclose(tt, 3 * ts.sum(axis=(1, 2)), rtol=1e-12)
+    assert np.allclose(tt + tv, 6 * len(pos), rtol=1e-12)
+
+
+def test_vv_statistic_is_tv_with_vision_rows_uniform_closed_form():
+    """VV budgeting takes the vision tokens' queries as the rows; under uniform
+    attention each vision row i puts |{j in V, j <= p_i}| / (p_i + 1) on vision keys."""
+    rng = np.random.default_rng(61)
+    modality = np.array([0, 0, 1, 1, 1, 0, 1, 1, 0], np.uint8)
+    vpos = np.flatnonzero(modality == 1)
+    L, H_q, d = 2, 3, 4
+    q = np.zeros((L, H_q, vpos.size, d))
+    k = rng.standard_normal((L, H_q, modality.size, d))
+    w = np.full((L, vpos.size), 1.0 / vpos.size)
+    _, vv = oracle.twr_scores_tvb_stat(q, k, modality, vpos, w, 1.0, H_q)
+    per_row = [np.count_nonzero(modality[:p + 1] == 1) / (p + 1) for p in vpos]
+    assert np.allclose(vv, H_q * sum(per_row), rtol=1e-13)
+
+
+def test_evict_budget_statistics():
+    rng = np.random.default_rng(62)
+    L, H_q, H_kv, d, n = 4, 4, 2, 8, 40
+    modality = np.zeros(n, np.uint8)
+    modality[6:30] = 1
+    pos = np.flatnonzero(modality == 0)[-8:]
+    qb = rng.integers(-2 ** 15, 2 ** 15, (L, H_q, pos.size, d)).astype(np.int16) & 0x3FFF
+    kb = rng.integers(-2 ** 15, 2 ** 15, (L, H_kv, n, d)).astype(np.int16) & 0x3FFF
+    vb = rng.integers(-2 ** 15, 2 ** 15, (L, H_kv, n, d)).astype(np.int16)
+    w = np.full((L, pos.size), 1.0 / pos.size)
+    total = oracle.vision_budget_total(0.3, 24, L)
+    ru = oracle.evict(qb, kb, vb, modality, pos, w, 0.3, H_kv, budget_stat="uniform")
+    assert ru["budgets"].tolist() == oracle.tvb_budgets(np.zeros(L), total, 24)
+    assert max(ru["budgets"]) - min(ru["budgets"]) <= 1
+    rt = oracle.evict(qb, kb, vb, modality, pos, w, 0.3, H_kv, budget_stat="tt")
+    q, k = oracle.widen_bf16(qb), oracle.widen_bf16(kb)
+    tt = oracle.tt_statistic(q, k, modality, pos, 1 / math.sqrt(d), H_kv)
+    assert np.array_equal(rt["stat"], tt)
+    assert rt["budgets"].tolist() == oracle.tvb_budgets(tt, total, 24)
