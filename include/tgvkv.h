@@ -52,6 +52,15 @@
  * (all-token basis) rows; sinks may add up to one row per sink per (l, g).
  * tgvkv_retained_rows gives the capacity, offsets[L*H_kv] the rows written.
  *
+ * Budget statistic (desc->budget_stat; the layer-budget policies of Table 1a
+ * and Eq. 5 with x in {VV, TV, TT}): TV (the method, default), TT (the
+ * text-text mass of the query rows; tgvkv_evict runs the text-key pass and
+ * returns that statistic in tvb_stat), or UNIFORM (no statistic).  VV, the
+ * vision-vision mass, needs the vision tokens' queries: call tgvkv_score with
+ * those queries as the rows (text_pos = the vision positions); its tvb_stat is
+ * then the VV statistic, to split with tgvkv_budget.  The TT statistic of a
+ * layer is also G * sum_{g,t} text_scores[l][g][t] (tgvkv_text_scores).
+ *
  * Text weights (desc->weight_mode): TGVKV_WEIGHTS_GIVEN uses the caller's w~
  * (Eq. 8); TGVKV_WEIGHTS_EQ7 makes tgvkv_evict derive w~ from the text-text
  * attention by Eq. 7 (tgvkv_text_scores) and ignore `w`.
@@ -87,6 +96,9 @@ extern "C" {
 #define TGVKV_BASIS_ALL     1   /* r counts all KV; both cases of Eq. 10 */
 #define TGVKV_WEIGHTS_GIVEN 0   /* the caller's normalised text weights w~ (default) */
 #define TGVKV_WEIGHTS_EQ7   1   /* tgvkv_evict derives w~ by Eq. 7 */
+#define TGVKV_STAT_TV       0   /* budgets follow the text-vision mass (Eq. 5, x = TV; default) */
+#define TGVKV_STAT_TT       1   /* ... the text-text mass (x = TT, Table 1a) */
+#define TGVKV_STAT_UNIFORM  2   /* ... no statistic: the uniform split of Table 1a */
 
 /* ---- problem description --------------------------------------------- */
 typedef struct tgvkv_desc {
@@ -104,6 +116,7 @@ typedef struct tgvkv_desc {
     int32_t weight_mode;    /* TGVKV_WEIGHTS_GIVEN (0) or TGVKV_WEIGHTS_EQ7 (tgvkv_evict) */
     int32_t keep_first;     /* sinks: the first keep_first positions are always kept */
     int32_t keep_last;      /* ... and the last keep_last positions */
+    int32_t budget_stat;    /* TGVKV_STAT_TV (0), TGVKV_STAT_TT or TGVKV_STAT_UNIFORM */
 } tgvkv_desc;
 
 /* Bytes of device workspace the calls below need for this problem. */
@@ -168,7 +181,8 @@ int tgvkv_text_scores(const tgvkv_desc* desc, const uint16_t* q_text, const uint
  * the largest fractional parts (ties: lower layer); a layer above N_v is capped
  * at N_v and the rest re-split over the other layers; all-zero statistics give a
  * uniform split.  The quotients are computed in double on the device.  Under
- * the all-token basis the same rule splits B with cap N.
+ * the all-token basis the same rule splits B with cap N.  With
+ * TGVKV_STAT_UNIFORM the statistic is not read (tvb_stat may be NULL).
  * tvb_stat: fp32 [L]; budgets: int32 [L] (output, rows per KV head: vision rows
  * under the vision basis, rows of any modality under the all-token basis). */
 int tgvkv_budget(const tgvkv_desc* desc, const float* tvb_stat, double ratio,

@@ -20,11 +20,12 @@ class Desc(ctypes.Structure):
                 ("N", c_int32), ("N_v", c_int32), ("n_win", c_int32),
                 ("softmax_scale", c_float), ("w_layer_stride", c_int64),
                 ("budget_basis", c_int32), ("weight_mode", c_int32),
-                ("keep_first", c_int32), ("keep_last", c_int32)]
+                ("keep_first", c_int32), ("keep_last", c_int32), ("budget_stat", c_int32)]
 
 
 BASIS_VISION, BASIS_ALL = 0, 1
 WEIGHTS_GIVEN, WEIGHTS_EQ7 = 0, 1
+STAT_TV, STAT_TT, STAT_UNIFORM = 0, 1, 2
 
 
 _P = ctypes.POINTER(Desc)

@@ -30,20 +30,22 @@ class TgvkvError(RuntimeError):
 
 BASIS = {"vision": _lib.BASIS_VISION, "all": _lib.BASIS_ALL}
 WEIGHTS = {"given": _lib.WEIGHTS_GIVEN, "eq7": _lib.WEIGHTS_EQ7}
+STAT = {"tv": _lib.STAT_TV, "tt": _lib.STAT_TT, "uniform": _lib.STAT_UNIFORM}
 
 
 def make_desc(L, H_q, H_kv, d, N, N_v, n_win, softmax_scale=0.0, w_layer_stride=None,
-              basis="vision", weights="given", keep_first=0, keep_last=0) -> Desc:
+              basis="vision", weights="given", keep_first=0, keep_last=0, stat="tv") -> Desc:
     """A problem descriptor; w_layer_stride defaults to n_win (one weight row per layer).
 
     basis: "vision" (r counts vision KV, every text KV kept) or "all" (r counts
     every KV, both cases of Eq. 10); weights: "given" (the caller's w~) or
-    "eq7" (tgvkv_evict derives w~ by Eq. 7); keep_first / keep_last: sinks."""
+    "eq7" (tgvkv_evict derives w~ by Eq. 7); keep_first / keep_last: sinks;
+    stat: the statistic the layer budgets follow, "tv" / "tt" / "uniform"."""
     return Desc(L=L, H_q=H_q, H_kv=H_kv, d=d, N=N, N_v=N_v, n_win=n_win,
                 softmax_scale=float(softmax_scale),
                 w_layer_stride=n_win if w_layer_stride is None else w_layer_stride,
                 budget_basis=BASIS[basis], weight_mode=WEIGHTS[weights],
-                keep_first=keep_first, keep_last=keep_last)
+                keep_first=keep_first, keep_last=keep_last, budget_stat=STAT[stat])
 
 
 def desc_for_workload(wl, softmax_scale=0.0, **options) -> Desc:

@@ -39,7 +39,9 @@ size_t round_up(size_t x) { return (x + 255) & ~size_t(255); }
 
 // tgvkv_evict needs the Eq. 9 text scores: for Eq. 7 weights, or for case
 // b_l <= N_t of Eq. 10 under the all-token basis.
-bool needs_text_pass(const Problem& p) { return p.weights_eq7 || p.basis == TGVKV_BASIS_ALL; }
+bool needs_text_pass(const Problem& p) {
+    return p.weights_eq7 || p.basis == TGVKV_BASIS_ALL || p.budget_stat == TGVKV_STAT_TT;
+}
 
 WsLayout layout_of(const Problem& p) {
     WsLayout w;
@@ -115,6 +117,10 @@ int make_problem(const tgvkv_desc* d, Problem* p) {
     p->weights_eq7 = d->weight_mode == TGVKV_WEIGHTS_EQ7;
     p->keep_first = d->keep_first < d->N ? d->keep_first : d->N;
     p->keep_last = d->keep_last < d->N ? d->keep_last : d->N;
+    if (d->budget_stat != TGVKV_STAT_TV && d->budget_stat != TGVKV_STAT_TT &&
+        d->budget_stat != TGVKV_STAT_UNIFORM)
+        return fail(TGVKV_ERR_INVALID_ARG, "budget_stat=%d unknown", d->budget_stat);
+    p->budget_stat = d->budget_stat;
     p->keys_text = 0;
     return TGVKV_OK;
 }
@@ -188,12 +194,12 @@ Problem text_problem(const Problem& p) {
 // Eq. 9 text scores and Eq. 7 weights: the text-key score pass, then the
 // per-layer weights.  stat_scratch takes the pass's (unused) statistic.
 int do_text_scores(const Problem& p, const uint16_t* q, const uint16_t* k, const uint8_t* modality,
-                   const int32_t* text_pos, float* text_scores, float* weights, float* stat_scratch,
-                   void* ws, cudaStream_t st) {
+                   const int32_t* text_pos, float* text_scores, float* weights, float* stat_out,
+                   void* ws, cudaStream_t st, long long budget_total = -1, int32_t* budgets = nullptr) {
     const WsLayout lay = layout_of(p);
     const Problem tp = text_problem(p);
-    cudaError_t e = launch_score(tp, q, k, modality, text_pos, nullptr, text_scores, stat_scratch,
-                                 static_cast<char*>(ws), lay, -1, nullptr, st);
+    cudaError_t e = launch_score(tp, q, k, modality, text_pos, nullptr, text_scores, stat_out,
+                                 static_cast<char*>(ws), lay, budget_total, budgets, st);
     if (e != cudaSuccess) return cuda_fail(e, "text-key score launch");
     if (weights) {
         e = launch_eq7_weights(p, text_scores, modality, text_pos, weights, status_of(ws, lay), st);
@@ -291,7 +297,7 @@ int tgvkv_budget(const tgvkv_desc* desc, const float* tvb_stat, double ratio, in
     int rc = make_problem(desc, &p);
     if (rc) return rc;
     if ((rc = check_ratio(ratio))) return rc;
-    REQUIRE_PTR(tvb_stat, "tvb_stat", false);
+    if (p.budget_stat != TGVKV_STAT_UNIFORM) REQUIRE_PTR(tvb_stat, "tvb_stat", false);
     REQUIRE_PTR(budgets, "budgets", false);
     REQUIRE_PTR(workspace, "workspace", true);
     const WsLayout lay = layout_of(p);
@@ -377,8 +383,12 @@ int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
         // Eq. 9 text scores (and Eq. 7 weights) into the workspace first
         text_scores = reinterpret_cast<float*>(wsb + lay.text_scores);
         float* wts = p.weights_eq7 ? reinterpret_cast<float*>(wsb + lay.weights) : nullptr;
+        // with TT budgeting the text pass's statistic (the text-text mass) is the one
+        // split, by that pass's last CTA
+        const bool tt = p.budget_stat == TGVKV_STAT_TT;
         rc = do_text_scores(p, q_text, k, modality, text_pos, text_scores, p.n_win > 0 ? wts : nullptr,
-                            reinterpret_cast<float*>(wsb + lay.stat_text), workspace, st);
+                            tt ? tvb_stat : reinterpret_cast<float*>(wsb + lay.stat_text), workspace, st,
+                            tt ? budget_total(p, ratio) : -1, tt ? budgets : nullptr);
         if (rc) return rc;
     }
     Problem ps = p;
@@ -387,9 +397,12 @@ int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
         w_used = reinterpret_cast<const float*>(wsb + lay.weights);
         ps.w_stride = p.n_win;
     }
-    // the score kernel's last CTA also derives the layer budgets
-    cudaError_t e = launch_score(ps, q_text, k, modality, text_pos, w_used, scores, tvb_stat,
-                                 wsb, lay, budget_total(p, ratio), budgets, st);
+    // the score kernel's last CTA also derives the layer budgets (TV or uniform;
+    // with TT budgeting the text pass did, and the TV statistic goes to scratch)
+    const bool tt = p.budget_stat == TGVKV_STAT_TT;
+    cudaError_t e = launch_score(ps, q_text, k, modality, text_pos, w_used, scores,
+                                 tt ? reinterpret_cast<float*>(wsb + lay.stat_text) : tvb_stat, wsb,
+                                 lay, budget_total(p, ratio), tt ? nullptr : budgets, st);
     if (e != cudaSuccess) return cuda_fail(e, "score launch");
     if (score_launches(p) == 0) {   // no score kernel ran: split the (zero) statistic here
         e = launch_budget(p, tvb_stat, budget_total(p, ratio), budgets, status, st);

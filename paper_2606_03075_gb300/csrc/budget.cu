@@ -9,10 +9,10 @@ namespace {
 constexpr int kThreads = 512;
 
 __global__ void __launch_bounds__(kThreads)
-tvb_budget_kernel(const float* __restrict__ stat, int L, long long total, int cap,
+tvb_budget_kernel(const float* __restrict__ stat, int L, long long total, int cap, int uniform,
                   int32_t* __restrict__ budgets, uint32_t* __restrict__ status) {
     __shared__ BudgetScratch scratch;
-    tvb_budget_block(stat, L, total, cap, budgets, status, scratch);
+    tvb_budget_block(stat, L, total, cap, budgets, status, scratch, uniform != 0);
 }
 
 }  // namespace
@@ -20,7 +20,8 @@ tvb_budget_kernel(const float* __restrict__ stat, int L, long long total, int ca
 cudaError_t launch_budget(const Problem& p, const float* tvb_stat, long long total,
                           int32_t* budgets, uint32_t* status, cudaStream_t stream) {
     const int cap = p.basis == TGVKV_BASIS_ALL ? p.N : p.N_v;
-    tvb_budget_kernel<<<1, kThreads, 0, stream>>>(tvb_stat, p.L, total, cap, budgets, status);
+    tvb_budget_kernel<<<1, kThreads, 0, stream>>>(tvb_stat, p.L, total, cap,
+                                                  p.budget_stat == TGVKV_STAT_UNIFORM, budgets, status);
     return cudaGetLastError();
 }
 

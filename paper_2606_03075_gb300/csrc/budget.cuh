@@ -28,13 +28,14 @@ struct BudgetScratch {
 // Every thread of the block must call this (it contains __syncthreads); every
 // block that calls it with the same statistic gets the same integers.
 // `stat` is read once into shared memory with L2-coherent loads.  When
-// `budgets` is null the result stays in b.result.
+// `budgets` is null the result stays in b.result.  `uniform` ignores the
+// statistic (the uniform budgeting of Table 1a: an all-zero statistic).
 __device__ __forceinline__ void tvb_budget_block(const float* stat, int L, long long total, int cap,
                                                  int32_t* budgets, uint32_t* status,
-                                                 BudgetScratch& b) {
+                                                 BudgetScratch& b, bool uniform = false) {
     const int tid = threadIdx.x, nt = blockDim.x;
     for (int l = tid; l < L; l += nt) {
-        b.stat[l] = (double)__ldcg(stat + l);
+        b.stat[l] = uniform ? 0.0 : (double)__ldcg(stat + l);
         b.active[l] = 1;
         b.result[l] = 0;
     }

@@ -1006,8 +1006,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
             __syncthreads();
             static_assert(sizeof(BudgetScratch) <= sizeof(s.k), "budget scratch in the K ring");
             tvb_budget_block(tvb_stat, p.L, budget_total, p.basis == TGVKV_BASIS_ALL ? p.N : p.N_v,
-                             budgets, status,
-                             *reinterpret_cast<BudgetScratch*>(&s.k[0][0][0]));
+                             budgets, status, *reinterpret_cast<BudgetScratch*>(&s.k[0][0][0]),
+                             p.budget_stat == TGVKV_STAT_UNIFORM);
         }
         if (tid == 0) *exit_counter = 0u;
     }

@@ -153,3 +153,15 @@ def test_decode_launch_count(lib):
                   w_layer_stride=wl.n_win)
         assert lib.tgvkv_decode_launches(ref(d)) == want[name], name
     assert lib.tgvkv_decode_launches(ref(_desc(d=48))) == -1
+
+
+def test_budget_statistic_modes(lib):
+    """TT budgeting runs the text-key pass (one more launch); uniform does not;
+    an unknown statistic is rejected."""
+    ref = ctypes.byref
+    wl = synth.WORKLOADS["llava15"]
+    base = dict(L=wl.L, H_q=wl.H_q, H_kv=wl.H_kv, d=wl.d, N=wl.N, N_v=wl.N_v, n_win=wl.n_win,
+                w_layer_stride=wl.n_win)
+    assert lib.tgvkv_evict_launches(ref(_desc(**base, budget_stat=1))) == 3
+    assert lib.tgvkv_evict_launches(ref(_desc(**base, budget_stat=2))) == 2
+    assert lib.tgvkv_evict_launches(ref(_desc(**base, budget_stat=3))) == -1

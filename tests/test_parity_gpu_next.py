@@ -327,3 +327,56 @@ def test_decode_empty_sets_give_zero(api):
     rows = torch.zeros((1, wl.d), dtype=torch.bfloat16, device="cuda")
     o = _run_decode(api, desc, _decode_q(wl, 9), rows, rows, offsets)
     assert np.array_equal(o, np.zeros_like(o))
+
+
+# ---------------------------------------------------------------- layer-budget statistics (Table 1a)
+@pytest.mark.parametrize("name", ["mha_single", "gqa_pairs", "text_heavy"])
+@pytest.mark.parametrize("stat", ["tt", "uniform"])
+def test_evict_budget_statistics(api, name, stat):
+    """TT budgets follow the text-key pass's text-text mass (returned as
+    tvb_stat); uniform budgets ignore the statistic.  Budgets exact given the
+    GPU statistic, the statistic within 1e-3, sets and rows exact."""
+    wl = CASES[name]
+    inp = synth.generate(wl, seed=10)
+    ratio = wl.ratios[0]
+    g = _evict(api, wl, inp, ratio, stat=stat)
+    assert g["status"] == 0
+    total = oracle.vision_budget_total(ratio, wl.N_v, wl.L)
+    if stat == "tt":
+        q, k = oracle.widen_bf16(inp["q"]), oracle.widen_bf16(inp["k"])
+        tt = oracle.tt_statistic(q, k, inp["modality"], inp["text_pos"], 1.0 / math.sqrt(wl.d),
+                                 wl.H_kv)
+        P.assert_close(g["stat"], tt, "TT statistic")
+        assert g["budgets"].tolist() == oracle.tvb_budgets(g["stat"], total, wl.N_v)
+    else:
+        assert g["budgets"].tolist() == oracle.tvb_budgets(np.zeros(wl.L), total, wl.N_v)
+    P.check_selection_and_compaction(wl, inp, g, list(range(wl.L)))
+
+
+def test_vv_statistic_with_vision_rows(api):
+    """VV budgeting: tgvkv_score with the vision tokens' queries as the rows
+    returns the vision-vision mass as tvb_stat; tgvkv_budget splits it."""
+    base = CASES["mha_single"]
+    vpos = np.flatnonzero(base.modality == 1)
+    rng = np.random.default_rng(11)
+    L, H_q, H_kv, d = base.L, base.H_q, base.H_kv, base.d
+    qv = synth.to_bf16_bits(rng.standard_normal((L, H_q, vpos.size, d)).astype(np.float32))
+    inp = synth.generate(base, seed=11)
+    desc = api.make_desc(L, H_q, H_kv, d, base.N, base.N_v, int(vpos.size))
+    ws = api.new_workspace(desc)
+    up = lambda a: torch.from_numpy(np.ascontiguousarray(a)).cuda()
+    w = torch.full((L, vpos.size), 1.0 / vpos.size, dtype=torch.float32, device="cuda")
+    sc = torch.empty((L, H_kv, base.N_v), dtype=torch.float32, device="cuda")
+    st = torch.empty(L, dtype=torch.float32, device="cuda")
+    api.tgvkv_score(desc, up(qv).view(torch.bfloat16), up(inp["k"]).view(torch.bfloat16),
+                    up(inp["modality"]), up(vpos.astype(np.int32)), w, sc, st, ws)
+    bud = torch.empty(L, dtype=torch.int32, device="cuda")
+    api.tgvkv_budget(desc, st, 0.2, bud, ws)
+    assert api.tgvkv_status(ws) == 0
+    _, vv = oracle.twr_scores_tvb_stat(oracle.widen_bf16(qv), oracle.widen_bf16(inp["k"]),
+                                       inp["modality"], vpos, np.full((L, vpos.size), 1.0 / vpos.size),
+                                       1.0 / math.sqrt(d), H_kv)
+    P.assert_close(st.cpu().numpy(), vv, "VV statistic")
+    assert bud.cpu().tolist() == oracle.tvb_budgets(st.cpu().numpy(),
+                                                    oracle.vision_budget_total(0.2, base.N_v, L),
+                                                    base.N_v)
