@@ -52,7 +52,12 @@ Beyond that hot path (same file, same conventions):
    ``S^TT_l = sum_{h,i} sum_{j in T} A_ij`` over the query rows; VV is the TV
    statistic of item 3 computed with the vision tokens' queries as the rows;
    uniform budgeting splits an all-zero statistic.
-13. Decode over the compacted cache (the consumer of the step, Section 3.1
+13. Head-adaptive budgets (an extension: the paper budgets per layer only,
+   Section 3.2): the statistic of a (layer, KV head) is the TV mass of its G
+   query heads; ``H_kv * B`` rows are split over the L * H_kv heads by the
+   same rule (cap N_v, or N under the all-token basis), and each head keeps its
+   own budget.
+14. Decode over the compacted cache (the consumer of the step, Section 3.1
    "Decode Phase"): a new token's query of head h attends to the retained
    rows of its KV head g = h // G, ``o = softmax(scale * q K_I^T) V_I``; a head
    with no retained row gives 0.
@@ -175,6 +180,26 @@ def text_scores_and_weights(q: np.ndarray, k: np.ndarray, modality: np.ndarray,
     return t_scores, weights
 
 
+def tv_statistic_per_head(q: np.ndarray, k: np.ndarray, modality: np.ndarray,
+                          text_pos: np.ndarray, scale: float, n_kv_heads: int) -> np.ndarray:
+    """[L, H_kv]: the TV mass (Eq. 5, x = TV) of the G query heads of each KV head."""
+    n_layers, n_q_heads = q.shape[0], q.shape[1]
+    group = n_q_heads // n_kv_heads
+    vision = np.flatnonzero(np.asarray(modality) == 1)
+    stat = np.zeros((n_layers, n_kv_heads))
+    for l in range(n_layers):
+        for h in range(n_q_heads):
+            a = causal_text_attention(q[l, h], k[l, h // group], text_pos, scale)
+            stat[l, h // group] += a[:, vision].sum()
+    return stat
+
+
+def head_budget(budgets, l: int, g: int) -> int:
+    """b of head (l, g): budgets is per layer [L] or per head [L, H_kv]."""
+    b = np.asarray(budgets)
+    return int(b[l]) if b.ndim == 1 else int(b[l, g])
+
+
 def tt_statistic(q: np.ndarray, k: np.ndarray, modality: np.ndarray, text_pos: np.ndarray,
                  scale: float, n_kv_heads: int) -> np.ndarray:
     """Eq. 5 with x = TT: per layer, the attention mass of the query rows on the
@@ -254,7 +279,7 @@ def tpr_select(scores: np.ndarray, budgets, modality: np.ndarray):
     """Retained positions per (layer, KV head) as CSR (offsets, idx).
 
     scores:  [L, H_kv, N_v] vision scores (any float precision).
-    budgets: [L] vision budget b_l of each layer.
+    budgets: [L] vision budget b_l of each layer, or [L, H_kv] one per head.
     Each set is all text positions plus the b_l vision positions ranked first
     by (score descending, position ascending), listed in ascending position
     order.  offsets has L*H_kv+1 entries, row-major over (layer, head).
@@ -269,7 +294,7 @@ def tpr_select(scores: np.ndarray, budgets, modality: np.ndarray):
         for g in range(n_kv_heads):
             s = scores[l, g]
             order = np.lexsort((np.arange(n_vision), -s))   # score desc, pos asc
-            chosen = vision[order[:int(budgets[l])]]
+            chosen = vision[order[:head_budget(budgets, l, g)]]
             rows = np.sort(np.concatenate([text, chosen]))
             kept.append(rows)
             offsets.append(offsets[-1] + rows.size)
@@ -311,8 +336,8 @@ def tpr_select_general(v_scores: np.ndarray, t_scores, budgets, modality: np.nda
     offsets = [0]
     kept = []
     for l in range(n_layers):
-        b = int(budgets[l])
         for g in range(n_kv_heads):
+            b = head_budget(budgets, l, g)
             if vision_basis or b > text.size:
                 slots = b if vision_basis else b - text.size
                 cand, s, always = vision, v_scores[l, g], text
@@ -390,7 +415,7 @@ def decode_attention(q: np.ndarray, k_rows: np.ndarray, v_rows: np.ndarray, offs
 def evict(q_bits, k_bits, v_bits, modality, text_pos, w, ratio: float,
           n_kv_heads: int, scale: float | None = None, weights: str = "given",
           basis: str = "vision", keep_first: int = 0, keep_last: int = 0,
-          budget_stat: str = "tv"):
+          budget_stat: str = "tv", head_budgets: bool = False):
     """Score, budget, select and compact, all in float64 on the host.
 
     weights: "given" uses ``w``; "eq7" derives w~ by Eq. 7 (``w`` is ignored).
@@ -399,6 +424,8 @@ def evict(q_bits, k_bits, v_bits, modality, text_pos, w, ratio: float,
              Eq. 10 applies per layer with the text scores of Eq. 9.
     budget_stat: the statistic the layer budgets follow: "tv" (the method),
              "tt" or "uniform" (Table 1a); the returned "stat" is the one split.
+    head_budgets: split H_kv * B over the (layer, KV head) pairs by their own TV
+             mass ("tv") or uniformly; budgets and stat are then [L, H_kv].
     """
     q = widen_bf16(q_bits)
     k = widen_bf16(k_bits)
@@ -416,13 +443,25 @@ def evict(q_bits, k_bits, v_bits, modality, text_pos, w, ratio: float,
             w = w_eq7
     w = np.asarray(w, dtype=np.float64)
     scores, stat = twr_scores_tvb_stat(q, k, modality, text_pos, w, scale, n_kv_heads)
-    if budget_stat == "tt":
+    if head_budgets:
+        if budget_stat == "tt":
+            raise ValueError("head budgets follow the TV mass or nothing")
+        stat = (np.zeros((n_layers, n_kv_heads)) if budget_stat == "uniform" else
+                tv_statistic_per_head(q, k, modality, text_pos, scale, n_kv_heads))
+    elif budget_stat == "tt":
         stat = tt_statistic(q, k, modality, text_pos, scale, n_kv_heads)
     elif budget_stat == "uniform":
         stat = np.zeros(n_layers)
+
+    def split(total, cap):
+        if not head_budgets:
+            return tvb_budgets(stat, total, cap)
+        return np.asarray(tvb_budgets(stat.ravel(), n_kv_heads * total, cap)).reshape(
+            n_layers, n_kv_heads)
+
     if basis == "vision":
         total = vision_budget_total(ratio, n_vision, n_layers)
-        budgets = tvb_budgets(stat, total, n_vision)
+        budgets = split(total, n_vision)
         if keep_first or keep_last:
             offsets, idx = tpr_select_general(scores, None, budgets, modality, keep_first,
                                               keep_last, vision_basis=True)
@@ -430,7 +469,7 @@ def evict(q_bits, k_bits, v_bits, modality, text_pos, w, ratio: float,
             offsets, idx = tpr_select(scores, budgets, modality)
     else:
         total = all_budget_total(ratio, n_tokens, n_layers)
-        budgets = tvb_budgets(stat, total, n_tokens)
+        budgets = split(total, n_tokens)
         offsets, idx = tpr_select_general(scores, t_scores, budgets, modality, keep_first,
                                           keep_last)
     k_out, v_out = compact(k_bits, v_bits, offsets, idx)

@@ -675,3 +675,49 @@ def test_evict_budget_statistics():
     tt = oracle.tt_statistic(q, k, modality, pos, 1 / math.sqrt(d), H_kv)
     assert np.array_equal(rt["stat"], tt)
     assert rt["budgets"].tolist() == oracle.tvb_budgets(tt, total, 24)
+
+
+# ---------------------------------------------------------------- head-adaptive budgets
+def test_per_head_tv_statistic_sums_to_layer_statistic():
+    q, k, modality, pos, w = _rand_case(L=3, H_q=6, H_kv=3, d=7, seed=70)
+    per_head = oracle.tv_statistic_per_head(q, k, modality, pos, 0.5, 3)
+    _, stat = oracle.twr_scores_tvb_stat(q, k, modality, pos, w, 0.5, 3)
+    assert np.allclose(per_head.sum(axis=1), stat, rtol=1e-12)
+    # one KV head per query head: each entry is that head's own TV mass
+    one = oracle.tv_statistic_per_head(q[:, :3], k, modality, pos, 0.5, 3)
+    for g in range(3):
+        _, sg = oracle.twr_scores_tvb_stat(q[:, g:g + 1], k[:, g:g + 1], modality, pos, w, 0.5, 1)
+        assert np.allclose(one[:, g], sg, rtol=1e-12)
+
+
+@pytest.mark.parametrize("basis", ["vision", "all"])
+@pytest.mark.parametrize("kind", ["tv", "uniform"])
+def test_evict_head_budgets(basis, kind):
+    """H_kv * B rows split over the heads; every head keeps its own count."""
+    rng = np.random.default_rng(71)
+    L, H_q, H_kv, d, n = 3, 4, 2, 8, 36
+    modality = np.zeros(n, np.uint8)
+    modality[5:28] = 1
+    pos = np.flatnonzero(modality == 0)[-6:]
+    qb = rng.integers(-2 ** 15, 2 ** 15, (L, H_q, pos.size, d)).astype(np.int16) & 0x3FFF
+    kb = rng.integers(-2 ** 15, 2 ** 15, (L, H_kv, n, d)).astype(np.int16) & 0x3FFF
+    vb = rng.integers(-2 ** 15, 2 ** 15, (L, H_kv, n, d)).astype(np.int16)
+    w = np.full((L, pos.size), 1.0 / pos.size)
+    r = oracle.evict(qb, kb, vb, modality, pos, w, 0.3, H_kv, basis=basis, budget_stat=kind,
+                     head_budgets=True)
+    b = r["budgets"]
+    assert b.shape == (L, H_kv)
+    total = (oracle.vision_budget_total(0.3, 23, L) if basis == "vision"
+             else oracle.all_budget_total(0.3, n, L))
+    assert int(b.sum()) == H_kv * total
+    if kind == "uniform":
+        assert b.max() - b.min() <= 1
+    else:
+        q, k = oracle.widen_bf16(qb), oracle.widen_bf16(kb)
+        st = oracle.tv_statistic_per_head(q, k, modality, pos, 1 / math.sqrt(d), H_kv)
+        assert np.array_equal(r["stat"], st)
+    n_t = n - 23
+    for l in range(L):
+        for g in range(H_kv):
+            cnt = r["offsets"][l * H_kv + g + 1] - r["offsets"][l * H_kv + g]
+            assert cnt == (n_t + b[l, g] if basis == "vision" else b[l, g])
