@@ -61,6 +61,13 @@
  * then the VV statistic, to split with tgvkv_budget.  The TT statistic of a
  * layer is also G * sum_{g,t} text_scores[l][g][t] (tgvkv_text_scores).
  *
+ * Head-adaptive budgets (desc->head_budgets = 1; an extension -- the paper
+ * budgets per layer only, Section 3.2): the statistic of (l, g) is the TV mass
+ * of its G query heads (tvb_stat[l*H_kv+g]), H_kv * B rows are split over the
+ * L * H_kv heads by the same rule (cap N_v, or N under the all-token basis),
+ * and set (l, g) keeps budgets[l*H_kv+g].  With TGVKV_STAT_UNIFORM the split
+ * is uniform over heads; TGVKV_STAT_TT is not supported.  At most 1024 heads.
+ *
  * Text weights (desc->weight_mode): TGVKV_WEIGHTS_GIVEN uses the caller's w~
  * (Eq. 8); TGVKV_WEIGHTS_EQ7 makes tgvkv_evict derive w~ from the text-text
  * attention by Eq. 7 (tgvkv_text_scores) and ignore `w`.
@@ -117,6 +124,8 @@ typedef struct tgvkv_desc {
     int32_t keep_first;     /* sinks: the first keep_first positions are always kept */
     int32_t keep_last;      /* ... and the last keep_last positions */
     int32_t budget_stat;    /* TGVKV_STAT_TV (0), TGVKV_STAT_TT or TGVKV_STAT_UNIFORM */
+    int32_t head_budgets;   /* 1: one budget per (layer, KV head); tvb_stat and budgets
+                               then hold L * H_kv entries (head-major within a layer) */
 } tgvkv_desc;
 
 /* Bytes of device workspace the calls below need for this problem. */
@@ -153,7 +162,8 @@ int64_t tgvkv_retained_rows(const tgvkv_desc* desc, double ratio);
  * text_pos: int32 [n_win], strictly ascending positions in [0, N)
  * w:        fp32 text weights w~ >= 0, row l at w + l * w_layer_stride, n_win floats
  * scores:   fp32 [L][H_kv][N_v]  (output)
- * tvb_stat: fp32 [L]             (output)
+ * tvb_stat: fp32 [L]             (output; [L][H_kv], the per-head masses, with
+ *           head budgets)
  * Arithmetic: bf16 products, fp32 accumulation and fp32 softmax. */
 int tgvkv_score(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* k,
                 const uint8_t* modality, const int32_t* text_pos, const float* w,

@@ -20,7 +20,8 @@ class Desc(ctypes.Structure):
                 ("N", c_int32), ("N_v", c_int32), ("n_win", c_int32),
                 ("softmax_scale", c_float), ("w_layer_stride", c_int64),
                 ("budget_basis", c_int32), ("weight_mode", c_int32),
-                ("keep_first", c_int32), ("keep_last", c_int32), ("budget_stat", c_int32)]
+                ("keep_first", c_int32), ("keep_last", c_int32), ("budget_stat", c_int32),
+                ("head_budgets", c_int32)]
 
 
 BASIS_VISION, BASIS_ALL = 0, 1

@@ -34,18 +34,27 @@ STAT = {"tv": _lib.STAT_TV, "tt": _lib.STAT_TT, "uniform": _lib.STAT_UNIFORM}
 
 
 def make_desc(L, H_q, H_kv, d, N, N_v, n_win, softmax_scale=0.0, w_layer_stride=None,
-              basis="vision", weights="given", keep_first=0, keep_last=0, stat="tv") -> Desc:
+              basis="vision", weights="given", keep_first=0, keep_last=0, stat="tv",
+              head_budgets=False) -> Desc:
     """A problem descriptor; w_layer_stride defaults to n_win (one weight row per layer).
 
     basis: "vision" (r counts vision KV, every text KV kept) or "all" (r counts
     every KV, both cases of Eq. 10); weights: "given" (the caller's w~) or
     "eq7" (tgvkv_evict derives w~ by Eq. 7); keep_first / keep_last: sinks;
-    stat: the statistic the layer budgets follow, "tv" / "tt" / "uniform"."""
+    stat: the statistic the layer budgets follow, "tv" / "tt" / "uniform";
+    head_budgets: one budget per (layer, KV head) (tvb_stat and budgets then
+    hold L * H_kv entries)."""
     return Desc(L=L, H_q=H_q, H_kv=H_kv, d=d, N=N, N_v=N_v, n_win=n_win,
                 softmax_scale=float(softmax_scale),
                 w_layer_stride=n_win if w_layer_stride is None else w_layer_stride,
                 budget_basis=BASIS[basis], weight_mode=WEIGHTS[weights],
-                keep_first=keep_first, keep_last=keep_last, budget_stat=STAT[stat])
+                keep_first=keep_first, keep_last=keep_last, budget_stat=STAT[stat],
+                head_budgets=int(bool(head_budgets)))
+
+
+def budget_units(desc: Desc) -> int:
+    """Entries of tvb_stat and budgets: L, or L * H_kv with head budgets."""
+    return desc.L * desc.H_kv if desc.head_budgets else desc.L
 
 
 def desc_for_workload(wl, softmax_scale=0.0, **options) -> Desc:
@@ -134,7 +143,7 @@ def tgvkv_score(desc, q_text, k, modality, text_pos, w, scores, tvb_stat, ws, st
         _ptr(text_pos, (torch.int32,), nw, "text_pos"),
         _ptr(w, (torch.float32,), wrows, "w"),
         _ptr(scores, (torch.float32,), L * Hkv * Nv, "scores"),
-        _ptr(tvb_stat, (torch.float32,), L, "tvb_stat"),
+        _ptr(tvb_stat, (torch.float32,), budget_units(desc), "tvb_stat"),
         _ptr(ws, (torch.uint8,), tgvkv_workspace_size(desc), "workspace"),
         _stream(stream)), "tgvkv_score")
 
@@ -156,8 +165,8 @@ def tgvkv_text_scores(desc, q_text, k, modality, text_pos, text_scores, weights,
 def tgvkv_budget(desc, tvb_stat, ratio, budgets, ws, stream=None):
     _check(_lib.load().tgvkv_budget(
         ctypes.byref(desc),
-        _ptr(tvb_stat, (torch.float32,), desc.L, "tvb_stat"), float(ratio),
-        _ptr(budgets, (torch.int32,), desc.L, "budgets"),
+        _ptr(tvb_stat, (torch.float32,), budget_units(desc), "tvb_stat"), float(ratio),
+        _ptr(budgets, (torch.int32,), budget_units(desc), "budgets"),
         _ptr(ws, (torch.uint8,), tgvkv_workspace_size(desc), "workspace"),
         _stream(stream)), "tgvkv_budget")
 
@@ -167,7 +176,7 @@ def tgvkv_select(desc, scores, budgets, modality, offsets, idx, ws, stream=None)
     _check(_lib.load().tgvkv_select(
         ctypes.byref(desc),
         _ptr(scores, (torch.float32,), LH * desc.N_v, "scores"),
-        _ptr(budgets, (torch.int32,), desc.L, "budgets"),
+        _ptr(budgets, (torch.int32,), budget_units(desc), "budgets"),
         _ptr(modality, (torch.uint8,), desc.N, "modality"),
         _ptr(offsets, (torch.int64,), LH + 1, "offsets"),
         _ptr(idx, (torch.int32,), 0, "idx"),
@@ -181,7 +190,7 @@ def tgvkv_select_tpr(desc, scores, text_scores, budgets, modality, offsets, idx,
         ctypes.byref(desc),
         _ptr(scores, (torch.float32,), LH * desc.N_v, "scores"),
         _ptr(text_scores, (torch.float32,), LH * (desc.N - desc.N_v), "text_scores"),
-        _ptr(budgets, (torch.int32,), desc.L, "budgets"),
+        _ptr(budgets, (torch.int32,), budget_units(desc), "budgets"),
         _ptr(modality, (torch.uint8,), desc.N, "modality"),
         _ptr(offsets, (torch.int64,), LH + 1, "offsets"),
         _ptr(idx, (torch.int32,), 0, "idx"),
@@ -218,8 +227,8 @@ def alloc_outputs(desc: Desc, ratio: float, device=None) -> EvictOutputs:
     L, Hkv = desc.L, desc.H_kv
     return EvictOutputs(
         scores=torch.empty((L, Hkv, desc.N_v), dtype=torch.float32, device=dev),
-        tvb_stat=torch.empty(L, dtype=torch.float32, device=dev),
-        budgets=torch.empty(L, dtype=torch.int32, device=dev),
+        tvb_stat=torch.empty(budget_units(desc), dtype=torch.float32, device=dev),
+        budgets=torch.empty(budget_units(desc), dtype=torch.int32, device=dev),
         offsets=torch.empty(L * Hkv + 1, dtype=torch.int64, device=dev),
         idx=torch.empty(max(rows, 1), dtype=torch.int32, device=dev),
         k_out=torch.empty((max(rows, 1), desc.d), dtype=torch.bfloat16, device=dev),
@@ -241,8 +250,8 @@ def tgvkv_evict(desc, q_text, k, v, modality, text_pos, w, ratio, out: EvictOutp
         _ptr(w, (torch.float32,), wrows, "w"),
         float(ratio),
         _ptr(out.scores, (torch.float32,), L * Hkv * Nv, "scores"),
-        _ptr(out.tvb_stat, (torch.float32,), L, "tvb_stat"),
-        _ptr(out.budgets, (torch.int32,), L, "budgets"),
+        _ptr(out.tvb_stat, (torch.float32,), budget_units(desc), "tvb_stat"),
+        _ptr(out.budgets, (torch.int32,), budget_units(desc), "budgets"),
         _ptr(out.offsets, (torch.int64,), L * Hkv + 1, "offsets"),
         _ptr(out.idx, (torch.int32,), rows, "idx"),
         _ptr(out.k_out, _BF16_LIKE, rows * d, "k_out"),

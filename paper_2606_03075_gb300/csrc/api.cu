@@ -121,6 +121,14 @@ int make_problem(const tgvkv_desc* d, Problem* p) {
         d->budget_stat != TGVKV_STAT_UNIFORM)
         return fail(TGVKV_ERR_INVALID_ARG, "budget_stat=%d unknown", d->budget_stat);
     p->budget_stat = d->budget_stat;
+    if (d->head_budgets != 0 && d->head_budgets != 1)
+        return fail(TGVKV_ERR_INVALID_ARG, "head_budgets=%d is neither 0 nor 1", d->head_budgets);
+    p->head_budgets = d->head_budgets;
+    if (p->head_budgets && p->budget_stat == TGVKV_STAT_TT)
+        return fail(TGVKV_ERR_UNSUPPORTED, "head budgets follow the TV mass or are uniform");
+    if (p->head_budgets && (long long)p->L * p->H_kv > kMaxL)
+        return fail(TGVKV_ERR_UNSUPPORTED, "head budgets for L * H_kv = %d heads above %d",
+                    p->L * p->H_kv, kMaxL);
     p->keys_text = 0;
     return TGVKV_OK;
 }
@@ -140,6 +148,11 @@ long long vision_budget_total(const Problem& p, double ratio) {
 long long budget_total(const Problem& p, double ratio) {
     if (p.basis == TGVKV_BASIS_ALL) return (long long)floor(ratio * (double)((long long)p.N * p.L) + 0.5);
     return vision_budget_total(p, ratio);
+}
+
+// Units the budget split shares out: per head, H_kv times the rows per head.
+long long split_total(const Problem& p, double ratio) {
+    return p.head_budgets ? (long long)p.H_kv * budget_total(p, ratio) : budget_total(p, ratio);
 }
 
 // The cap of one layer's budget in the split.
@@ -301,7 +314,7 @@ int tgvkv_budget(const tgvkv_desc* desc, const float* tvb_stat, double ratio, in
     REQUIRE_PTR(budgets, "budgets", false);
     REQUIRE_PTR(workspace, "workspace", true);
     const WsLayout lay = layout_of(p);
-    cudaError_t e = launch_budget(p, tvb_stat, budget_total(p, ratio), budgets,
+    cudaError_t e = launch_budget(p, tvb_stat, split_total(p, ratio), budgets,
                                   status_of(workspace, lay), static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? ok() : cuda_fail(e, "budget launch");
 }
@@ -388,7 +401,7 @@ int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
         const bool tt = p.budget_stat == TGVKV_STAT_TT;
         rc = do_text_scores(p, q_text, k, modality, text_pos, text_scores, p.n_win > 0 ? wts : nullptr,
                             tt ? tvb_stat : reinterpret_cast<float*>(wsb + lay.stat_text), workspace, st,
-                            tt ? budget_total(p, ratio) : -1, tt ? budgets : nullptr);
+                            tt ? split_total(p, ratio) : -1, tt ? budgets : nullptr);
         if (rc) return rc;
     }
     Problem ps = p;
@@ -402,10 +415,10 @@ int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
     const bool tt = p.budget_stat == TGVKV_STAT_TT;
     cudaError_t e = launch_score(ps, q_text, k, modality, text_pos, w_used, scores,
                                  tt ? reinterpret_cast<float*>(wsb + lay.stat_text) : tvb_stat, wsb,
-                                 lay, budget_total(p, ratio), tt ? nullptr : budgets, st);
+                                 lay, split_total(p, ratio), tt ? nullptr : budgets, st);
     if (e != cudaSuccess) return cuda_fail(e, "score launch");
     if (score_launches(p) == 0) {   // no score kernel ran: split the (zero) statistic here
-        e = launch_budget(p, tvb_stat, budget_total(p, ratio), budgets, status, st);
+        e = launch_budget(p, tvb_stat, split_total(p, ratio), budgets, status, st);
         if (e != cudaSuccess) return cuda_fail(e, "budget launch");
     }
     e = launch_select_compact(p, scores, text_scores, budgets, modality, offsets, idx, k, v, k_out,

@@ -20,7 +20,8 @@ tvb_budget_kernel(const float* __restrict__ stat, int L, long long total, int ca
 cudaError_t launch_budget(const Problem& p, const float* tvb_stat, long long total,
                           int32_t* budgets, uint32_t* status, cudaStream_t stream) {
     const int cap = p.basis == TGVKV_BASIS_ALL ? p.N : p.N_v;
-    tvb_budget_kernel<<<1, kThreads, 0, stream>>>(tvb_stat, p.L, total, cap,
+    const int units = p.head_budgets ? p.L * p.H_kv : p.L;
+    tvb_budget_kernel<<<1, kThreads, 0, stream>>>(tvb_stat, units, total, cap,
                                                   p.budget_stat == TGVKV_STAT_UNIFORM, budgets, status);
     return cudaGetLastError();
 }

@@ -19,6 +19,7 @@ struct Problem {
     int weights_eq7;       // tgvkv_evict derives w~ by Eq. 7
     int keep_first, keep_last;   // sink tokens, clipped to [0, N]
     int budget_stat;       // statistic the budgets split: TGVKV_STAT_TV / _TT / _UNIFORM
+    int head_budgets;      // one budget per (layer, KV head) instead of per layer
     // Score kernel only: the key set of pass B.  0 = vision keys (Eq. 8, row
     // weights w~); 1 = text keys with unit row weights (Eq. 9).  N_v then
     // holds the size of that key set, N_t; the launcher sets both.

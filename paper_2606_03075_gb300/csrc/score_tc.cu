@@ -996,16 +996,22 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
     __syncthreads();
     if (s.cta_last) {
         __threadfence();
-        for (int l = tid; l < p.L; l += NTHREADS) {
-            float S = 0.f;
-            for (int g = 0; g < p.H_kv; ++g) S += __ldcg(&stat_head[(size_t)l * p.H_kv + g]);
-            tvb_stat[l] = S;
+        if (p.head_budgets) {
+            // head-adaptive budgets: the statistic is the TV mass of each (layer, KV head)
+            for (int lh = tid; lh < p.L * p.H_kv; lh += NTHREADS) tvb_stat[lh] = __ldcg(&stat_head[lh]);
+        } else {
+            for (int l = tid; l < p.L; l += NTHREADS) {
+                float S = 0.f;
+                for (int g = 0; g < p.H_kv; ++g) S += __ldcg(&stat_head[(size_t)l * p.H_kv + g]);
+                tvb_stat[l] = S;
+            }
         }
         if (budgets) {
-            // the layer budgets of Eq. 5, with the now idle K ring as scratch
+            // the budgets of Eq. 5, with the now idle K ring as scratch
             __syncthreads();
             static_assert(sizeof(BudgetScratch) <= sizeof(s.k), "budget scratch in the K ring");
-            tvb_budget_block(tvb_stat, p.L, budget_total, p.basis == TGVKV_BASIS_ALL ? p.N : p.N_v,
+            tvb_budget_block(tvb_stat, p.head_budgets ? p.L * p.H_kv : p.L, budget_total,
+                             p.basis == TGVKV_BASIS_ALL ? p.N : p.N_v,
                              budgets, status, *reinterpret_cast<BudgetScratch*>(&s.k[0][0][0]),
                              p.budget_stat == TGVKV_STAT_UNIFORM);
         }
@@ -1116,7 +1122,8 @@ cudaError_t launch_score(const Problem& p, const uint16_t* q, const uint16_t* k,
         cudaError_t e = cudaSuccess;
         if (p.N_v > 0)
             e = cudaMemsetAsync(scores, 0, sizeof(float) * (size_t)p.L * p.H_kv * p.N_v, stream);
-        if (e == cudaSuccess) e = cudaMemsetAsync(tvb_stat, 0, sizeof(float) * (size_t)p.L, stream);
+        const size_t units = p.head_budgets ? (size_t)p.L * p.H_kv : (size_t)p.L;
+        if (e == cudaSuccess) e = cudaMemsetAsync(tvb_stat, 0, sizeof(float) * units, stream);
         return e;
     }
     if (p.d == 64)

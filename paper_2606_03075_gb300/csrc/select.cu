@@ -484,14 +484,34 @@ tpr_select_general_kernel(Problem p, const float* __restrict__ scores,
     __syncthreads();
     const int sink_v = s_sink_v, sink_t = s_sink_t;
     const int cap = budget_cap_of(p);
-    int b = budgets[l];
+    int b = budgets[p.head_budgets ? lg : l];
     if (b < 0 || b > cap) {
         if (tid == 0) raise_status(status, TGVKV_STATUS_BUDGET);
         b = b < 0 ? 0 : cap;
     }
     const TprCase c = tpr_case(p, b, sink_v, sink_t);
     const int len = c.len;
-    if (tid == 0) {
+    if (p.head_budgets) {
+        // CSR offset: the set sizes of every earlier head, summed by the block
+        long long part = 0;
+        for (int m = tid; m < lg; m += kThreads) {
+            int bm = budgets[m];
+            bm = bm < 0 ? 0 : (bm > cap ? cap : bm);
+            part += tpr_case(p, bm, sink_v, sink_t).len;
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(~0u, part, o);
+        __shared__ long long warp_part[kThreads / 32];
+        if (lane == 0) warp_part[warp] = part;
+        __syncthreads();
+        if (tid == 0) {
+            long long off = 0;
+            for (int w = 0; w < kThreads / 32; ++w) off += warp_part[w];
+            s_off = off;
+            offsets[lg] = off;
+            if (lg == p.L * p.H_kv - 1) offsets[lg + 1] = off + len;
+        }
+    } else if (tid == 0) {
         long long off = 0;
         for (int m = 0; m < l; ++m) {
             int bm = budgets[m];
@@ -673,7 +693,7 @@ cudaError_t launch_sel_general(const Problem& p, const float* scores, const floa
 
 // The hot-path kernels cover the vision basis without sinks.
 inline bool general_select(const Problem& p) {
-    return p.basis == TGVKV_BASIS_ALL || p.keep_first > 0 || p.keep_last > 0;
+    return p.basis == TGVKV_BASIS_ALL || p.keep_first > 0 || p.keep_last > 0 || p.head_budgets;
 }
 
 // Warps per CTA of the warp-per-head kernel for p (0: use the CTA-per-head

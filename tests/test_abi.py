@@ -165,3 +165,19 @@ def test_budget_statistic_modes(lib):
     assert lib.tgvkv_evict_launches(ref(_desc(**base, budget_stat=1))) == 3
     assert lib.tgvkv_evict_launches(ref(_desc(**base, budget_stat=2))) == 2
     assert lib.tgvkv_evict_launches(ref(_desc(**base, budget_stat=3))) == -1
+
+
+def test_head_budget_options(lib):
+    ref = ctypes.byref
+    wl = synth.WORKLOADS["llava15"]
+    base = dict(L=wl.L, H_q=wl.H_q, H_kv=wl.H_kv, d=wl.d, N=wl.N, N_v=wl.N_v, n_win=wl.n_win,
+                w_layer_stride=wl.n_win)
+    # same capacity as per-layer budgets: H_kv * B rows are shared out either way
+    for r in (0.05, 0.2):
+        assert (lib.tgvkv_retained_rows(ref(_desc(**base, head_budgets=1)), r) ==
+                lib.tgvkv_retained_rows(ref(_desc(**base)), r))
+    assert lib.tgvkv_evict_launches(ref(_desc(**base, head_budgets=1))) == 2
+    assert lib.tgvkv_evict_launches(ref(_desc(**base, head_budgets=1, budget_stat=1))) == -1
+    assert lib.tgvkv_evict_launches(ref(_desc(**base, head_budgets=2))) == -1
+    big = dict(base, L=64, H_q=32, H_kv=32)            # 2048 heads
+    assert lib.tgvkv_evict_launches(ref(_desc(**big, head_budgets=1))) == -1

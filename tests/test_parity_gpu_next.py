@@ -380,3 +380,37 @@ def test_vv_statistic_with_vision_rows(api):
     assert bud.cpu().tolist() == oracle.tvb_budgets(st.cpu().numpy(),
                                                     oracle.vision_budget_total(0.2, base.N_v, L),
                                                     base.N_v)
+
+
+# ---------------------------------------------------------------- head-adaptive budgets
+@pytest.mark.parametrize("name", ["mha_single", "gqa_pairs", "mha_packed_d64"])
+@pytest.mark.parametrize("basis,stat", [("vision", "tv"), ("all", "tv"), ("vision", "uniform")])
+def test_evict_head_budgets(api, name, basis, stat):
+    """One budget per (layer, KV head): the per-head TV masses within 1e-3,
+    budgets exact from the GPU's masses, sets and rows exact."""
+    wl = CASES[name]
+    inp = synth.generate(wl, seed=12)
+    ratio = 0.3 if basis == "all" else wl.ratios[0]
+    g = _evict(api, wl, inp, ratio, basis=basis, stat=stat, head_budgets=True)
+    assert g["status"] == 0
+    L, H = wl.L, wl.H_kv
+    if basis == "all":
+        total, cap = oracle.all_budget_total(ratio, wl.N, L), wl.N
+    else:
+        total, cap = oracle.vision_budget_total(ratio, wl.N_v, L), wl.N_v
+    stat_used = g["stat"] if stat == "tv" else np.zeros(L * H)
+    if stat == "tv":
+        q, k = oracle.widen_bf16(inp["q"]), oracle.widen_bf16(inp["k"])
+        ref = oracle.tv_statistic_per_head(q, k, inp["modality"], inp["text_pos"],
+                                           1.0 / math.sqrt(wl.d), H)
+        P.assert_close(g["stat"].reshape(L, H), ref, "per-head TV mass")
+    budgets = np.asarray(oracle.tvb_budgets(stat_used, H * total, cap)).reshape(L, H)
+    np.testing.assert_array_equal(g["budgets"].reshape(L, H), budgets)
+    ts = _run_text(api, wl, g["dev"])[0] if basis == "all" else None
+    off, idx = oracle.tpr_select_general(g["scores"], ts, budgets, inp["modality"],
+                                         vision_basis=basis == "vision")
+    np.testing.assert_array_equal(g["offsets"], off)
+    np.testing.assert_array_equal(g["idx"], idx)
+    ko, vo = oracle.compact(inp["k"], inp["v"], off, idx)
+    np.testing.assert_array_equal(g["k_out"], ko)
+    np.testing.assert_array_equal(g["v_out"], vo)
