@@ -87,21 +87,30 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
         b = b < 0 ? 0 : p.N_v;
     }
     const int len = p.N_t + b;
-    if (tid == 0) {
-        long long off = 0;
-        for (int m = 0; m < l; ++m) {
+    // CSR offset: the sets of the earlier layers, summed by the whole block
+    // (their budgets load in parallel, not one after another)
+    __shared__ long long off_part[kThreads / 32];
+    {
+        long long part = 0;
+        for (int m = tid; m < l; m += kThreads) {
             int bm = budgets[m];
             bm = bm < 0 ? 0 : (bm > p.N_v ? p.N_v : bm);
-            off += (long long)p.H_kv * (p.N_t + bm);
+            part += (long long)p.H_kv * (p.N_t + bm);
         }
-        off += (long long)g * len;
-        s_off = off;
-        offsets[lg] = off;
-        if (lg == p.L * p.H_kv - 1) offsets[lg + 1] = off + len;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(~0u, part, o);
+        if (lane == 0) off_part[warp] = part;
     }
     const float* sc = scores + (size_t)lg * p.N_v;
     for (int i = tid; i < p.N_v; i += kThreads) keys[i] = float_order_key(__ldg(sc + i));
     __syncthreads();
+    if (tid == 0) {
+        long long off = (long long)g * len;
+        for (int w = 0; w < kThreads / 32; ++w) off += off_part[w];
+        s_off = off;
+        offsets[lg] = off;
+        if (lg == p.L * p.H_kv - 1) offsets[lg + 1] = off + len;
+    }
 
     // ---- radix select of the b-th largest key
     uint32_t prefix = 0;
@@ -511,17 +520,26 @@ tpr_select_general_kernel(Problem p, const float* __restrict__ scores,
             offsets[lg] = off;
             if (lg == p.L * p.H_kv - 1) offsets[lg + 1] = off + len;
         }
-    } else if (tid == 0) {
-        long long off = 0;
-        for (int m = 0; m < l; ++m) {
+    } else {
+        // the sets of the earlier layers, summed by the whole block
+        long long part = 0;
+        for (int m = tid; m < l; m += kThreads) {
             int bm = budgets[m];
             bm = bm < 0 ? 0 : (bm > cap ? cap : bm);
-            off += (long long)p.H_kv * tpr_case(p, bm, sink_v, sink_t).len;
+            part += (long long)p.H_kv * tpr_case(p, bm, sink_v, sink_t).len;
         }
-        off += (long long)g * len;
-        s_off = off;
-        offsets[lg] = off;
-        if (lg == p.L * p.H_kv - 1) offsets[lg + 1] = off + len;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(~0u, part, o);
+        __shared__ long long layer_part[kThreads / 32];
+        if (lane == 0) layer_part[warp] = part;
+        __syncthreads();
+        if (tid == 0) {
+            long long off = (long long)g * len;
+            for (int w = 0; w < kThreads / 32; ++w) off += layer_part[w];
+            s_off = off;
+            offsets[lg] = off;
+            if (lg == p.L * p.H_kv - 1) offsets[lg + 1] = off + len;
+        }
     }
     const int n_cand = c.vision ? p.N_v : p.N_t;
     const uint8_t cand_mod = c.vision ? 1 : 0;
