@@ -57,10 +57,11 @@ WsLayout layout_of(const Problem& p) {
     w.decode_part = o;
     if (decode_splits(p) > 1)
         o += round_up(sizeof(float) * (size_t)p.L * p.H_q * decode_splits(p) * (p.d + 2));
-    w.text_scores = w.weights = 0;
+    w.text_scores = w.weights = w.row_stats = 0;
     if (needs_text_pass(p)) {
         w.text_scores = o; o += round_up(sizeof(float) * (size_t)p.L * p.H_kv * (p.N_t > 0 ? p.N_t : 1));
         w.weights = o;     o += round_up(sizeof(float) * (size_t)p.L * (p.n_win > 0 ? p.n_win : 1));
+        w.row_stats = o;   o += round_up(3 * sizeof(float) * ((size_t)p.L * p.H_q * p.n_win + 1));
     }
     w.total = o;
     return w;
@@ -130,6 +131,8 @@ int make_problem(const tgvkv_desc* d, Problem* p) {
         return fail(TGVKV_ERR_UNSUPPORTED, "head budgets for L * H_kv = %d heads above %d",
                     p->L * p->H_kv, kMaxL);
     p->keys_text = 0;
+    p->row_stats = nullptr;
+    p->stats_given = 0;
     return TGVKV_OK;
 }
 
@@ -208,9 +211,11 @@ Problem text_problem(const Problem& p) {
 // per-layer weights.  stat_scratch takes the pass's (unused) statistic.
 int do_text_scores(const Problem& p, const uint16_t* q, const uint16_t* k, const uint8_t* modality,
                    const int32_t* text_pos, float* text_scores, float* weights, float* stat_out,
-                   void* ws, cudaStream_t st, long long budget_total = -1, int32_t* budgets = nullptr) {
+                   void* ws, cudaStream_t st, long long budget_total = -1, int32_t* budgets = nullptr,
+                   float* row_stats = nullptr) {
     const WsLayout lay = layout_of(p);
-    const Problem tp = text_problem(p);
+    Problem tp = text_problem(p);
+    tp.row_stats = row_stats;
     cudaError_t e = launch_score(tp, q, k, modality, text_pos, nullptr, text_scores, stat_out,
                                  static_cast<char*>(ws), lay, budget_total, budgets, st);
     if (e != cudaSuccess) return cuda_fail(e, "text-key score launch");
@@ -401,10 +406,17 @@ int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
         const bool tt = p.budget_stat == TGVKV_STAT_TT;
         rc = do_text_scores(p, q_text, k, modality, text_pos, text_scores, p.n_win > 0 ? wts : nullptr,
                             tt ? tvb_stat : reinterpret_cast<float*>(wsb + lay.stat_text), workspace, st,
-                            tt ? split_total(p, ratio) : -1, tt ? budgets : nullptr);
+                            tt ? split_total(p, ratio) : -1, tt ? budgets : nullptr,
+                            reinterpret_cast<float*>(wsb + lay.row_stats));
         if (rc) return rc;
     }
     Problem ps = p;
+    if (needs_text_pass(p)) {
+        // the vision pass takes the rows' (m, Z, vision mass) from the text-key
+        // pass instead of a pass A of its own
+        ps.row_stats = reinterpret_cast<float*>(wsb + lay.row_stats);
+        ps.stats_given = 1;
+    }
     const float* w_used = w;
     if (p.weights_eq7) {
         w_used = reinterpret_cast<const float*>(wsb + lay.weights);

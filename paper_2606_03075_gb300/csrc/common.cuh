@@ -24,6 +24,11 @@ struct Problem {
     // weights w~); 1 = text keys with unit row weights (Eq. 9).  N_v then
     // holds the size of that key set, N_t; the launcher sets both.
     int keys_text;
+    // Row statistics (m, Z, vision mass) per global query row, float [3 * L*H_q*n_win]:
+    // the text-key pass writes them when not null; with stats_given the vision
+    // pass reads them and skips its pass A (tgvkv_evict with a text-key pass).
+    float* row_stats;
+    int stats_given;
 };
 
 // Row splits of the decode kernel: enough CTAs for two per SM on the 152 SMs
@@ -53,6 +58,7 @@ struct WsLayout {
     size_t text_scores; // float [L*H_kv*N_t]: Eq. 9 scores
     size_t weights;     // float [L*n_win]: Eq. 7 weights
     size_t stat_text;   // float [L]: the text-key pass's (unused) statistic
+    size_t row_stats;   // float [3*L*H_q*n_win]: per-row (m, Z, vision mass) of the text-key pass
     size_t decode_part; // float [L*H_q*S*(d+2)]: decode row-split partials (S > 1)
     size_t total;
 };

@@ -98,9 +98,10 @@ struct PSmem {
     int vq[MAXT][4];                         // vision keys before each 32-key word
     int rt_max[MAX_RT], rt_min[MAX_RT];      // per row tile: max / min query position
     alignas(16) int row_pos[2][BM];          // per row slot and TMEM lane: position, -1 = none
+    int row_q[2][BM];                        // ... its global Q row, -1 = none
     alignas(16) float row_nmp[2][BM];        // -(m_i - log2 c_i); -inf = no row
     float row_w[2][BM], row_mass[2][BM];
-    float part_m[4][BM], part_z[4][BM], part_v[4][BM];
+    float part_m[4][BM], part_z[4][BM], part_v[4][BM], part_u[4][BM];
     int item_q[NIQ];
     uint32_t tmem_base;
     int abort_flag, never, stop, head_last, cur_item, cta_last;
@@ -187,7 +188,8 @@ __device__ __forceinline__ Item item_info(const Problem& p, const PSmem<D>& s, i
 // kt[1] is the second tile of a single step or the second head's tile of a
 // packed step (-1: none); pair steps use kt[0] for both row tiles.
 __device__ __forceinline__ bool next_step(const Item& it, int mode, int pass, int& cur,
-                                          const int* vis_before, int (&kt)[2]) {
+                                          const int* vis_before, int (&kt)[2], bool stats_given) {
+    if (pass == 0 && stats_given) return false;   // the row statistics come from the workspace
     int c = pass == 0 ? cur : next_vis_tile(vis_before, cur, it.ntmax);
     if (c >= it.ntmax) return false;
     kt[0] = c;
@@ -279,7 +281,56 @@ __device__ __forceinline__ void exp_word(const float (&x)[32], float sl2, float 
     }
 }
 
+// exp_word plus the sum over the visible keys NOT in vm (u): the text-key pass
+// keeps the vision mass of each row this way, for the vision pass to reuse.
+template <bool MASKED>
+__device__ __forceinline__ void exp_word_both(const float (&x)[32], float sl2, float nm, int lim,
+                                              uint32_t vm, float& z, float& v, float& u) {
+    if (vm == 0u || vm == 0xFFFFFFFFu) {
+        float zs = 0.f;
+        exp_word<MASKED>(x, sl2, nm, lim, 0u, zs, zs);   // (v untouched when vm == 0)
+        z += zs;
+        if (vm) v += zs;
+        else u += zs;
+    } else {
+        const float2 s2 = make_float2(sl2, sl2), n2 = make_float2(nm, nm);
+        float2 za = make_float2(0.f, 0.f), va = za, ua = za;
+#pragma unroll
+        for (int c = 0; c < 32; c += 2) {
+            const float2 t = fma2(make_float2(x[c], x[c + 1]), s2, n2);
+            float2 e = make_float2(fast_exp2(t.x), fast_exp2(t.y));
+            if (MASKED) {
+                if (c > lim) e.x = 0.f;
+                if (c + 1 > lim) e.y = 0.f;
+            }
+            za = add2(za, e);
+            const bool b0 = (vm >> c) & 1u, b1 = (vm >> (c + 1)) & 1u;
+            va = add2(va, make_float2(b0 ? e.x : 0.f, b1 ? e.y : 0.f));
+            ua = add2(ua, make_float2(b0 ? 0.f : e.x, b1 ? 0.f : e.y));
+        }
+        z += za.x + za.y;
+        v += va.x + va.y;
+        u += ua.x + ua.y;
+    }
+}
+
 // Online statistics of one row over one 32-key word: columns 0..lim visible.
+// row_word with the complement mass u as well (text-key pass).
+__device__ __forceinline__ void row_word_both(const float (&x)[32], float sl2, int lim, uint32_t vm,
+                                              float& m, float& z, float& v, float& u) {
+    if (lim < 0) return;
+    const float m_new = fmaxf(m, (lim >= 31 ? max32(x) : max32_masked(x, lim)) * sl2);
+    const float alpha = fast_exp2(m - m_new);
+    z *= alpha;
+    v *= alpha;
+    u *= alpha;
+    if (lim >= 31)
+        exp_word_both<false>(x, sl2, -m_new, 31, vm, z, v, u);
+    else
+        exp_word_both<true>(x, sl2, -m_new, lim, vm, z, v, u);
+    m = m_new;
+}
+
 __device__ __forceinline__ void row_word(const float (&x)[32], float sl2, int lim, uint32_t vm,
                                          float& m, float& z, float& v) {
     if (lim < 0) return;
@@ -372,6 +423,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
                 float* __restrict__ score_part, float* __restrict__ stat_part,
                 float* __restrict__ stat_head, uint32_t* __restrict__ tickets,
                 uint32_t* __restrict__ status, long long budget_total, int32_t* __restrict__ budgets) {
+    float* row_stats = p.row_stats;
     extern __shared__ unsigned char smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     PSmem<D>& s = *reinterpret_cast<PSmem<D>*>(smem_raw + (((raw + 1023u) & ~1023u) - raw));
@@ -560,7 +612,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
             };
             for (int pass = 0; ok && pass < 2; ++pass) {
                 int cur = 0, kt[2];
-                while (ok && next_step(itm, mode, pass, cur, s.vis_before, kt)) {
+                while (ok && next_step(itm, mode, pass, cur, s.vis_before, kt, p.stats_given)) {
                     load(itm.lh[0], kt[0]);
                     if (ok && kt[1] >= 0)
                         load(mode == MODE_PACKED ? itm.lh[1] : itm.lh[0], kt[1]);
@@ -616,7 +668,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
             const uint64_t qd = qdesc0 + (uint64_t)(qs0 * Q_SLOT);
             for (int pass = 0; ok && pass < 2; ++pass) {
                 int cur = 0, kt[2];
-                while (ok && next_step(itm, mode, pass, cur, s.vis_before, kt)) {
+                while (ok && next_step(itm, mode, pass, cur, s.vis_before, kt, p.stats_given)) {
                     // pair steps take one stage; single and packed steps two (an even
                     // pair of adjacent stages), the second possibly unused
                     const int nst = mode == MODE_PAIR ? 1 : 2;
@@ -739,6 +791,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
                 }
                 s.row_pos[rs][ln] = pos;
                 s.row_w[rs][ln] = wr;
+                s.row_q[rs][ln] = has ? Item::pick(itm.qy, part) + row : -1;
             }
             // the item's output rows start at zero: pass B adds two partial sums per key
             for (int r = 0; r < itm.nparts; ++r) {
@@ -755,13 +808,13 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
             // packed: head b = quarter >> 1, columns 128b + 32 wi + [0, 32)
             const int rsA = mode == MODE_PAIR ? (wi >> 1) : 0;
             const int my_pos = s.row_pos[rsA][ln];
-            float m = -INFINITY, z = 0.f, v = 0.f;
+            float m = -INFINITY, z = 0.f, v = 0.f, u = 0.f;
             {
                 // Every warp runs every step of the item, also after a failed wait
                 // (then doing nothing), so that the warps of a quarter always meet
                 // at the same named barriers.
                 int cur = 0, kt[2];
-                while (next_step(itm, mode, 0, cur, s.vis_before, kt)) {
+                while (next_step(itm, mode, 0, cur, s.vis_before, kt, p.stats_given)) {
                     const int b = step & 1;
                     ++step;
                     if (ok && !warp_wait(&s.s_full[b], ((step - 1) >> 1) & 1, abort_flag)) {
@@ -801,7 +854,11 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
                             tc::tmem_wait_ld();
                             if (ch == nch - 1) release_acc(&s.s_empty[b], lane);
                             const int lim = my_pos - (ktile * BN + cbase + ch * 32);
-                            row_word(x, sl2, lim, s.vmask[ktile][(cbase >> 5) + ch], m, z, v);
+                            const uint32_t vm = s.vmask[ktile][(cbase >> 5) + ch];
+                            if (p.keys_text)   // also the vision mass, for the vision pass
+                                row_word_both(x, sl2, lim, vm, m, z, v, u);
+                            else
+                                row_word(x, sl2, lim, vm, m, z, v);
                         }
                     }
                 }
@@ -811,20 +868,38 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
             s.part_m[wi][ln] = m;
             s.part_z[wi][ln] = z;
             s.part_v[wi][ln] = v;
+            s.part_u[wi][ln] = u;
             tc::named_bar_sync(2 + quarter, 128);
             // pair: warps 0 and 2 combine parts {0,1} / {2,3} of row slot 0 / 1;
             // single and packed: warp 0 combines all four
             if (mode == MODE_PAIR ? ((wi & 1) == 0 && (wi >> 1) < itm.nparts) : wi == 0) {
                 const int rs = mode == MODE_PAIR ? (wi >> 1) : 0;
                 const int c0 = mode == MODE_PAIR ? wi : 0, c1 = mode == MODE_PAIR ? wi + 2 : 4;
+                const int qr = s.row_q[rs][ln];
                 float mt = -INFINITY;
-                for (int c = c0; c < c1; ++c) mt = fmaxf(mt, s.part_m[c][ln]);
                 float zt = 0.f, vt = 0.f;
-                if (mt != -INFINITY) {
-                    for (int c = c0; c < c1; ++c) {
-                        const float a = fast_exp2(s.part_m[c][ln] - mt);
-                        zt += s.part_z[c][ln] * a;
-                        vt += s.part_v[c][ln] * a;
+                if (p.stats_given) {
+                    // (m, Z, vision mass) of the row, from the text-key pass
+                    if (qr >= 0) {
+                        mt = __ldcg(row_stats + 3 * (size_t)qr);
+                        zt = __ldcg(row_stats + 3 * (size_t)qr + 1);
+                        vt = __ldcg(row_stats + 3 * (size_t)qr + 2);
+                    }
+                } else {
+                    for (int c = c0; c < c1; ++c) mt = fmaxf(mt, s.part_m[c][ln]);
+                    float ut = 0.f;
+                    if (mt != -INFINITY) {
+                        for (int c = c0; c < c1; ++c) {
+                            const float a = fast_exp2(s.part_m[c][ln] - mt);
+                            zt += s.part_z[c][ln] * a;
+                            vt += s.part_v[c][ln] * a;
+                            ut += s.part_u[c][ln] * a;
+                        }
+                    }
+                    if (p.keys_text && row_stats && qr >= 0) {
+                        row_stats[3 * (size_t)qr] = mt;
+                        row_stats[3 * (size_t)qr + 1] = zt;
+                        row_stats[3 * (size_t)qr + 2] = ut;
                     }
                 }
                 const bool valid = s.row_pos[rs][ln] >= 0 && zt > 0.f;
@@ -864,7 +939,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
             // Pair items write one partial row per row tile.
             {
                 int cur = 0, kt[2];
-                while (next_step(itm, mode, 1, cur, s.vis_before, kt)) {
+                while (next_step(itm, mode, 1, cur, s.vis_before, kt, p.stats_given)) {
                     const int b = step & 1;
                     if (ok && !warp_wait(&s.s_full[b], (step >> 1) & 1, abort_flag)) {
                         ok = false;
