@@ -414,3 +414,40 @@ def test_evict_head_budgets(api, name, basis, stat):
     ko, vo = oracle.compact(inp["k"], inp["v"], off, idx)
     np.testing.assert_array_equal(g["k_out"], ko)
     np.testing.assert_array_equal(g["v_out"], vo)
+
+
+def test_widened_paths_back_to_back_stay_clean(api):
+    """Many consecutive calls of the widened evict paths and of decode on one
+    workspace: the status stays clean and every call gives the first call's
+    result bit for bit (the text-key pass hands row statistics to the vision
+    pass through the workspace each time)."""
+    wl = CASES["gqa_pairs"]
+    inp = synth.generate(wl, seed=13)
+    dev = P.device_inputs(inp)
+    for opts in (dict(weights="eq7"), dict(basis="all", keep_first=4, keep_last=1),
+                 dict(stat="tt", head_budgets=False), dict(head_budgets=True)):
+        desc = api.desc_for_workload(wl, **opts)
+        ws = api.new_workspace(desc)
+        out = api.alloc_outputs(desc, wl.ratios[0])
+        w = None if opts.get("weights") == "eq7" else dev["w"]
+        first = None
+        for it in range(40):
+            api.tgvkv_evict(desc, dev["q"], dev["k"], dev["v"], dev["modality"], dev["text_pos"], w,
+                            wl.ratios[0], out, ws)
+            if it in (0, 39):
+                assert api.tgvkv_status(ws) == 0, opts
+                n = int(out.offsets[-1].item())
+                snap = (out.scores.cpu().numpy().copy(), out.idx[:n].cpu().numpy().copy())
+                if first is None:
+                    first = snap
+                else:
+                    np.testing.assert_array_equal(snap[0], first[0])
+                    np.testing.assert_array_equal(snap[1], first[1])
+        qd = torch.from_numpy(_decode_q(wl, 14)).cuda().view(torch.bfloat16)
+        o1 = torch.empty((wl.L, wl.H_q, wl.d), dtype=torch.float32, device="cuda")
+        o2 = torch.empty_like(o1)
+        api.tgvkv_decode(desc, qd, out.k_out, out.v_out, out.offsets, o1, ws)
+        for _ in range(20):
+            api.tgvkv_decode(desc, qd, out.k_out, out.v_out, out.offsets, o2, ws)
+        assert api.tgvkv_status(ws) == 0
+        assert torch.equal(o1, o2)
