@@ -12,7 +12,7 @@ What is computed, in the paper's order (Section 3.3, "TGV-KV"):
    ``j <= p_i`` (every modality); keys after p_i are masked with -inf.
 2. Text-Vision attention (Eq. 6): the columns of those rows that belong to
    vision keys.  This is read as a *slice* of the full causal softmax (the
-   paper slices A^(TV) "out of A_l"), not as a softmax restricted to vision
+   paper takes A^(TV) as a block of A_l), not as a softmax restricted to vision
    keys.
 3. TVB statistic (Eq. 5 with x = TV): ``S_l = sum_{h,i,j in V} A_ij`` over all
    query heads of layer l.
