@@ -8,4 +8,5 @@ from .tgvkv_oracle import (  # noqa: F401
     tvb_budgets, tpr_select, compact, compacted_kv_bytes, evict,
     text_scores_and_weights, all_budget_total, sink_positions, tpr_select_general,
     decode_attention, tt_statistic, tv_statistic_per_head, head_budget,
+    prefill_attention, row_statistics,
 )

@@ -61,6 +61,12 @@ Beyond that hot path (same file, same conventions):
    "Decode Phase"): a new token's query of head h attends to the retained
    rows of its KV head g = h // G, ``o = softmax(scale * q K_I^T) V_I``; a head
    with no retained row gives 0.
+15. Prefill attention and the row statistics it leaves (the producer side of
+   the step, Section 3.1 "Prefill Phase" with Eq. 2 over every row): each
+   token i attends causally to the keys j <= i, ``o_i = sum_j A_ij v_j``; at
+   the query positions p_i the rows' log-normaliser and vision mass
+   ``sum_{j in V} A_ij`` are what Eq. 5 / Eq. 6 need, so a prefill that keeps
+   them spares the eviction step its own pass over the row statistics.
 
 Floating point: inputs are bf16 bit patterns widened exactly to float64; all
 arithmetic is float64.  The paper states no precision.
@@ -407,6 +413,64 @@ def decode_attention(q: np.ndarray, k_rows: np.ndarray, v_rows: np.ndarray, offs
             e = np.exp(logits - logits.max())
             out[l, h] = (e / e.sum()) @ v_rows[lo:hi]
     return out
+
+
+# --------------------------------------------------------------------------
+# Prefill attention over every token, and the row statistics it leaves
+# --------------------------------------------------------------------------
+def prefill_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float,
+                      n_kv_heads: int):
+    """Causal attention of every token of the prefill (Eq. 2 for all N rows,
+    then the attention-weighted sum of the value rows).
+
+    q: [L, H_q, N, d] float64 queries of every token; k, v: [L, H_kv, N, d].
+    Returns (o, bound), both [L, H_q, N, d], with g = h // G:
+      o[l, h, i]     = sum_{j <= i} A_ij v[l, g, j],  A_i = softmax_j(scale <q_i, k_j>)
+      bound[l, h, i] = sum_{j <= i} A_ij |v[l, g, j]|  (the size of the terms, which
+                       sets how far a rounded computation of o may stray)
+    """
+    n_layers, n_q_heads, n, _ = q.shape
+    group = n_q_heads // n_kv_heads
+    visible = np.tril(np.ones((n, n), dtype=bool))     # key j visible from row i iff j <= i
+    o = np.zeros_like(q)
+    bound = np.zeros_like(q)
+    for l in range(n_layers):
+        for h in range(n_q_heads):
+            g = h // group
+            logits = np.where(visible, scale * (q[l, h] @ k[l, g].T), -np.inf)
+            e = np.exp(logits - logits.max(axis=1, keepdims=True))
+            a = e / e.sum(axis=1, keepdims=True)
+            o[l, h] = a @ v[l, g]
+            bound[l, h] = a @ np.abs(v[l, g])
+    return o, bound
+
+
+def row_statistics(q: np.ndarray, k: np.ndarray, modality: np.ndarray, text_pos: np.ndarray,
+                   scale: float, n_kv_heads: int):
+    """The eviction step's per-row quantities at the query positions (Eq. 2, 5, 6).
+
+    q: [L, H_q, N, d] float64 queries of every token; the query row i of the
+    step is the token at position p_i = text_pos[i].  k: [L, H_kv, N, d].
+    Returns (lse2, vision), both [L, H_q, n_win]:
+      lse2[l, h, i]   = log2 sum_{j <= p_i} exp(scale <q_{p_i}, k_j>)
+      vision[l, h, i] = sum_{j <= p_i, j vision} A_ij  (the row's share of Eq. 6)
+    """
+    n_layers, n_q_heads, n, _ = q.shape
+    group = n_q_heads // n_kv_heads
+    pos = np.asarray(text_pos, dtype=np.int64)
+    is_vision = np.asarray(modality) == 1
+    lse2 = np.zeros((n_layers, n_q_heads, pos.size))
+    vision = np.zeros((n_layers, n_q_heads, pos.size))
+    for l in range(n_layers):
+        for h in range(n_q_heads):
+            logits = scale * (q[l, h, pos] @ k[l, h // group].T)
+            logits = np.where(np.arange(n)[None, :] <= pos[:, None], logits, -np.inf)
+            top = logits.max(axis=1)
+            e = np.exp(logits - top[:, None])
+            z = e.sum(axis=1)
+            lse2[l, h] = (top + np.log(z)) / math.log(2.0)
+            vision[l, h] = e[:, is_vision].sum(axis=1) / z
+    return lse2, vision
 
 
 # --------------------------------------------------------------------------

@@ -721,3 +721,85 @@ def test_evict_head_budgets(basis, kind):
         for g in range(H_kv):
             cnt = r["offsets"][l * H_kv + g + 1] - r["offsets"][l * H_kv + g]
             assert cnt == (n_t + b[l, g] if basis == "vision" else b[l, g])
+
+
+# ---------------------------------------------------------------- prefill attention and its row statistics
+def _prefill_case(L=2, H_q=4, H_kv=2, n=11, d=5, seed=70):
+    rng = np.random.default_rng(seed)
+    q = rng.standard_normal((L, H_q, n, d))
+    k = rng.standard_normal((L, H_kv, n, d))
+    v = rng.standard_normal((L, H_kv, n, d))
+    return q, k, v
+
+
+def test_prefill_attention_brute_force():
+    """Eq. 2 over every row, term by term with scalar exponentials, then A V;
+    G = 2, so query heads 2g and 2g+1 read KV head g."""
+    q, k, v = _prefill_case()
+    L, H_q, n, d = q.shape
+    scale = 0.41
+    o, bound = oracle.prefill_attention(q, k, v, scale, 2)
+    for l in range(L):
+        for h in range(H_q):
+            g = h // 2
+            for i in range(n):
+                x = [scale * sum(q[l, h, i, c] * k[l, g, j, c] for c in range(d)) for j in range(i + 1)]
+                top = max(x)
+                e = [math.exp(t - top) for t in x]
+                z = sum(e)
+                for c in range(d):
+                    ref = sum(e[j] / z * v[l, g, j, c] for j in range(i + 1))
+                    mag = sum(e[j] / z * abs(v[l, g, j, c]) for j in range(i + 1))
+                    assert abs(o[l, h, i, c] - ref) <= 1e-12 * (1 + abs(ref))
+                    assert abs(bound[l, h, i, c] - mag) <= 1e-12 * (1 + mag)
+
+
+def test_prefill_attention_closed_forms():
+    """Rows of A sum to 1: equal value rows come back unchanged.  Q = 0: every
+    visible key gets 1/(i + 1), so o_i is the running mean of v_0..v_i."""
+    q, k, v = _prefill_case(L=1, H_q=3, H_kv=3, n=9, d=4, seed=71)
+    const = np.broadcast_to(np.array([0.5, -2.0, 3.25, 0.0]), v.shape).copy()
+    o, bound = oracle.prefill_attention(q, k, const, 0.9, 3)
+    assert np.allclose(o, const, rtol=0, atol=1e-14)
+    assert np.allclose(bound, np.abs(const), rtol=0, atol=1e-14)
+    o, _ = oracle.prefill_attention(np.zeros_like(q), k, v, 0.9, 3)
+    running = np.cumsum(v, axis=2) / np.arange(1, 10)[None, None, :, None]
+    assert np.allclose(o, running, rtol=1e-13, atol=1e-15)
+    # the first token sees only itself
+    o, _ = oracle.prefill_attention(q, k, v, 0.9, 3)
+    assert np.allclose(o[:, :, 0], v[:, :, 0], rtol=0, atol=1e-15)
+
+
+def test_prefill_rows_at_query_positions_match_eviction_rows():
+    """The prefill rows at the query positions are the eviction step's rows of
+    Eq. 2 (the separately written causal_text_attention), times V."""
+    q, k, v = _prefill_case(L=2, H_q=6, H_kv=2, n=12, d=4, seed=72)
+    pos = np.array([3, 7, 8, 11])
+    o, _ = oracle.prefill_attention(q, k, v, 0.7, 2)
+    for l in range(2):
+        for h in range(6):
+            a = oracle.causal_text_attention(q[l, h, pos], k[l, h // 3], pos, 0.7)
+            assert np.allclose(o[l, h, pos], a @ v[l, h // 3], rtol=1e-12, atol=1e-14)
+
+
+def test_row_statistics_closed_form_and_eq5():
+    """Q = 0: log2 of p_i + 1 visible unit terms, and the vision share is the
+    fraction of vision keys among them.  Random Q: the vision shares summed over
+    query heads and rows are the TVB statistic S_l of Eq. 5."""
+    q, k, modality, pos, w = _rand_case(L=3, H_q=6, H_kv=2, d=7, seed=73)
+    n = modality.size
+    rng = np.random.default_rng(74)
+    q_all = rng.standard_normal((3, 6, n, 7))
+    q_all[:, :, pos] = q                       # the query rows sit at their positions
+    lse2, vis = oracle.row_statistics(np.zeros_like(q_all), k, modality, pos, 0.6, 2)
+    for i, p in enumerate(pos):
+        assert np.allclose(lse2[:, :, i], math.log2(p + 1), rtol=0, atol=1e-13)
+        assert np.allclose(vis[:, :, i], np.count_nonzero(modality[: p + 1] == 1) / (p + 1),
+                           rtol=1e-13)
+    lse2, vis = oracle.row_statistics(q_all, k, modality, pos, 0.6, 2)
+    _, stat = oracle.twr_scores_tvb_stat(q, k, modality, pos, w, 0.6, 2)
+    assert np.allclose(vis.sum(axis=(1, 2)), stat, rtol=1e-12)
+    # lse2 against a direct log-sum-exp of one row
+    l, h, i = 1, 4, 2
+    x = [0.6 * float(q[l, h, i] @ k[l, h // 3, j]) for j in range(pos[i] + 1)]
+    assert abs(lse2[l, h, i] - math.log2(sum(math.exp(t) for t in x))) < 1e-12
