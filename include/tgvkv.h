@@ -237,6 +237,46 @@ int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
                 int64_t* offsets, int32_t* idx, uint16_t* k_out, uint16_t* v_out,
                 void* workspace, void* stream);
 
+/* Causal prefill attention over every token, which also keeps what the
+ * eviction step needs from the rows at its query positions (the prefill phase
+ * of Section 3.1: Eq. 2 over all N rows; Eq. 5 / Eq. 6 read the same rows).
+ *
+ * For every layer l, query head h (KV head g = h / G) and token i:
+ *   o[l][h][i][:] = sum_{j <= i} softmax_j(softmax_scale <q[l][h][i], k[l][g][j]>) v[l][g][j][:]
+ * and for every query row r of the eviction step (position p = text_pos[r]):
+ *   q_text[l][h][r][:]  = q[l][h][p][:]                      (bit copy)
+ *   row_stats[l][h][r]  = (m, Z, V):  Z = sum_{j <= p} 2^(x_pj log2(e) - m),
+ *                         V = the same sum over the vision keys j,
+ *                         x_pj = softmax_scale <q[l][h][p], k[l][g][j]>,
+ *                         m = a reference value at most 8 below the row's
+ *                         largest x_pj log2(e) and not above it.
+ * q: bf16 [L][H_q][N][d]; k, v: bf16 [L][H_kv][N][d]; modality: uint8 [N];
+ * text_pos: int32 [n_win] strictly ascending (may be NULL when n_win = 0);
+ * o: bf16 [L][H_q][N][d] (output); q_text: bf16 [L][H_q][n_win][d] (output);
+ * row_stats: fp32 [L][H_q][n_win][3] (output).  q, k, v, o and q_text must be
+ * 16-byte aligned.  bf16 products with fp32 accumulation and softmax; the
+ * attention weights enter the value product rounded to bf16, and o is rounded
+ * to bf16.  q_text and row_stats are the inputs tgvkv_evict_with_stats takes.
+ * Device-side checks: text_pos (TGVKV_STATUS_TEXT_POS), bounded waits
+ * (TGVKV_STATUS_TIMEOUT). */
+int tgvkv_prefill(const tgvkv_desc* desc, const uint16_t* q, const uint16_t* k,
+                  const uint16_t* v, const uint8_t* modality, const int32_t* text_pos,
+                  uint16_t* o, uint16_t* q_text, float* row_stats, void* workspace,
+                  void* stream);
+
+/* tgvkv_evict with the query rows' statistics given: row_stats as tgvkv_prefill
+ * writes them (fp32 [L][H_q][n_win][3]).  The score passes then read each
+ * row's (m, Z, vision mass) instead of streaming its keys a first time; all
+ * other arguments and every result are those of tgvkv_evict.  Budgets by the
+ * TT statistic need each row's text mass, which row_stats does not hold:
+ * TGVKV_ERR_UNSUPPORTED. */
+int tgvkv_evict_with_stats(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* k,
+                           const uint16_t* v, const uint8_t* modality, const int32_t* text_pos,
+                           const float* w, double ratio, const float* row_stats,
+                           float* scores, float* tvb_stat, int32_t* budgets,
+                           int64_t* offsets, int32_t* idx, uint16_t* k_out, uint16_t* v_out,
+                           void* workspace, void* stream);
+
 /* Number of CUDA kernels one tgvkv_evict call launches for this problem
  * (introspection for callers that budget launches, e.g. inside a captured
  * graph; the paper has no counterpart): normally 2 (scores with the layer

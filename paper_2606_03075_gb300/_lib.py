@@ -51,6 +51,12 @@ SIGNATURES = {
     "tgvkv_evict": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                             c_double, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                             c_void_p, c_void_p, c_void_p, c_void_p]),
+    "tgvkv_evict_with_stats": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                       c_void_p, c_double, c_void_p, c_void_p, c_void_p,
+                                       c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                       c_void_p, c_void_p]),
+    "tgvkv_prefill": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                              c_void_p, c_void_p, c_void_p, c_void_p]),
     "tgvkv_workspace_init": (c_int, [_P, c_void_p, c_void_p]),
     "tgvkv_status": (c_int, [c_void_p, c_void_p]),
     "tgvkv_evict_launches": (c_int, [_P]),

@@ -260,6 +260,51 @@ def tgvkv_evict(desc, q_text, k, v, modality, text_pos, w, ratio, out: EvictOutp
         _stream(stream)), "tgvkv_evict")
 
 
+def tgvkv_evict_with_stats(desc, q_text, k, v, modality, text_pos, w, ratio, row_stats,
+                           out: EvictOutputs, ws, stream=None):
+    """tgvkv_evict with the query rows' (m, Z, vision mass) from tgvkv_prefill."""
+    L, Hq, Hkv, d, N, Nv, nw = desc.L, desc.H_q, desc.H_kv, desc.d, desc.N, desc.N_v, desc.n_win
+    rows = tgvkv_retained_rows(desc, ratio)
+    wrows = (L - 1) * desc.w_layer_stride + nw if nw else 0
+    _check(_lib.load().tgvkv_evict_with_stats(
+        ctypes.byref(desc),
+        _ptr(q_text, _BF16_LIKE, L * Hq * nw * d, "q_text"),
+        _ptr(k, _BF16_LIKE, L * Hkv * N * d, "k"),
+        _ptr(v, _BF16_LIKE, L * Hkv * N * d, "v"),
+        _ptr(modality, (torch.uint8,), N, "modality"),
+        _ptr(text_pos, (torch.int32,), nw, "text_pos"),
+        _ptr(w, (torch.float32,), wrows, "w"),
+        float(ratio),
+        _ptr(row_stats, (torch.float32,), 3 * L * Hq * nw, "row_stats"),
+        _ptr(out.scores, (torch.float32,), L * Hkv * Nv, "scores"),
+        _ptr(out.tvb_stat, (torch.float32,), budget_units(desc), "tvb_stat"),
+        _ptr(out.budgets, (torch.int32,), budget_units(desc), "budgets"),
+        _ptr(out.offsets, (torch.int64,), L * Hkv + 1, "offsets"),
+        _ptr(out.idx, (torch.int32,), rows, "idx"),
+        _ptr(out.k_out, _BF16_LIKE, rows * d, "k_out"),
+        _ptr(out.v_out, _BF16_LIKE, rows * d, "v_out"),
+        _ptr(ws, (torch.uint8,), tgvkv_workspace_size(desc), "workspace"),
+        _stream(stream)), "tgvkv_evict_with_stats")
+
+
+def tgvkv_prefill(desc, q, k, v, modality, text_pos, o, q_text, row_stats, ws, stream=None):
+    """Causal prefill attention over every token, plus the eviction step's query
+    rows (q_text) and their (m, Z, vision mass) (see include/tgvkv.h)."""
+    L, Hq, Hkv, d, N, nw = desc.L, desc.H_q, desc.H_kv, desc.d, desc.N, desc.n_win
+    _check(_lib.load().tgvkv_prefill(
+        ctypes.byref(desc),
+        _ptr(q, _BF16_LIKE, L * Hq * N * d, "q"),
+        _ptr(k, _BF16_LIKE, L * Hkv * N * d, "k"),
+        _ptr(v, _BF16_LIKE, L * Hkv * N * d, "v"),
+        _ptr(modality, (torch.uint8,), N, "modality"),
+        _ptr(text_pos, (torch.int32,), nw, "text_pos"),
+        _ptr(o, _BF16_LIKE, L * Hq * N * d, "o"),
+        _ptr(q_text, _BF16_LIKE, L * Hq * nw * d, "q_text"),
+        _ptr(row_stats, (torch.float32,), 3 * L * Hq * nw, "row_stats"),
+        _ptr(ws, (torch.uint8,), tgvkv_workspace_size(desc), "workspace"),
+        _stream(stream)), "tgvkv_prefill")
+
+
 def tgvkv_status(ws: torch.Tensor, stream=None) -> int:
     """Synchronise the stream, return and clear the device status bits."""
     rc = _lib.load().tgvkv_status(_ptr(ws, (torch.uint8,), 4, "workspace"), _stream(stream))

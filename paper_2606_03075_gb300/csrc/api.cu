@@ -212,10 +212,11 @@ Problem text_problem(const Problem& p) {
 int do_text_scores(const Problem& p, const uint16_t* q, const uint16_t* k, const uint8_t* modality,
                    const int32_t* text_pos, float* text_scores, float* weights, float* stat_out,
                    void* ws, cudaStream_t st, long long budget_total = -1, int32_t* budgets = nullptr,
-                   float* row_stats = nullptr) {
+                   float* row_stats = nullptr, bool stats_given = false) {
     const WsLayout lay = layout_of(p);
     Problem tp = text_problem(p);
     tp.row_stats = row_stats;
+    tp.stats_given = stats_given ? 1 : 0;
     cudaError_t e = launch_score(tp, q, k, modality, text_pos, nullptr, text_scores, stat_out,
                                  static_cast<char*>(ws), lay, budget_total, budgets, st);
     if (e != cudaSuccess) return cuda_fail(e, "text-key score launch");
@@ -241,6 +242,82 @@ int check_score_args(const Problem& p, const uint16_t* q, const uint16_t* k,
     REQUIRE_PTR(tvb_stat, "tvb_stat", false);
     REQUIRE_PTR(ws, "workspace", true);
     return TGVKV_OK;
+}
+
+// tgvkv_evict, with the query rows' (m, Z, vision mass) computed by the score
+// passes, or given by the caller (stats_given).
+int evict_impl(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* k,
+               const uint16_t* v, const uint8_t* modality, const int32_t* text_pos,
+               const float* w, double ratio, bool stats_given, const float* given_stats, float* scores,
+               float* tvb_stat, int32_t* budgets, int64_t* offsets, int32_t* idx, uint16_t* k_out,
+               uint16_t* v_out, void* workspace, void* stream) {
+    Problem p{};
+    int rc = make_problem(desc, &p);
+    if (rc) return rc;
+    if ((rc = check_ratio(ratio))) return rc;
+    if (stats_given && p.budget_stat == TGVKV_STAT_TT)
+        return fail(TGVKV_ERR_UNSUPPORTED,
+                    "TT budgets need the rows' text mass, which the given statistics do not hold");
+    if (stats_given && p.n_win > 0) REQUIRE_PTR(given_stats, "row_stats", false);
+    // with no query rows (n_win = 0) no score pass runs and nothing is read
+    float* stats = stats_given && p.n_win > 0 ? const_cast<float*>(given_stats) : nullptr;
+    rc = check_score_args(p, q_text, k, modality, text_pos, w, scores, tvb_stat, workspace,
+                          !p.weights_eq7);
+    if (rc) return rc;
+    REQUIRE_PTR(v, "v", true);
+    REQUIRE_PTR(budgets, "budgets", false);
+    REQUIRE_PTR(offsets, "offsets", false);
+    REQUIRE_PTR(idx, "idx", false);
+    REQUIRE_PTR(k_out, "k_out", true);
+    REQUIRE_PTR(v_out, "v_out", true);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const WsLayout lay = layout_of(p);
+    uint32_t* status = status_of(workspace, lay);
+    char* wsb = static_cast<char*>(workspace);
+    float* text_scores = nullptr;
+    if (needs_text_pass(p)) {
+        // Eq. 9 text scores (and Eq. 7 weights) into the workspace first
+        text_scores = reinterpret_cast<float*>(wsb + lay.text_scores);
+        float* wts = p.weights_eq7 ? reinterpret_cast<float*>(wsb + lay.weights) : nullptr;
+        // with TT budgeting the text pass's statistic (the text-text mass) is the one
+        // split, by that pass's last CTA
+        const bool tt = p.budget_stat == TGVKV_STAT_TT;
+        // the text-key pass computes the rows' (m, Z, vision mass) into the
+        // workspace, or reads the given ones
+        rc = do_text_scores(p, q_text, k, modality, text_pos, text_scores, p.n_win > 0 ? wts : nullptr,
+                            tt ? tvb_stat : reinterpret_cast<float*>(wsb + lay.stat_text), workspace, st,
+                            tt ? split_total(p, ratio) : -1, tt ? budgets : nullptr,
+                            stats ? stats : reinterpret_cast<float*>(wsb + lay.row_stats),
+                            stats != nullptr);
+        if (rc) return rc;
+    }
+    Problem ps = p;
+    if (stats || needs_text_pass(p)) {
+        // the vision pass takes the rows' (m, Z, vision mass) from the caller or
+        // the text-key pass instead of a pass A of its own
+        ps.row_stats = stats ? stats : reinterpret_cast<float*>(wsb + lay.row_stats);
+        ps.stats_given = 1;
+    }
+    const float* w_used = w;
+    if (p.weights_eq7) {
+        w_used = reinterpret_cast<const float*>(wsb + lay.weights);
+        ps.w_stride = p.n_win;
+    }
+    // the score kernel's last CTA also derives the layer budgets (TV or uniform;
+    // with TT budgeting the text pass did, and the TV statistic goes to scratch)
+    const bool tt = p.budget_stat == TGVKV_STAT_TT;
+    cudaError_t e = launch_score(ps, q_text, k, modality, text_pos, w_used, scores,
+                                 tt ? reinterpret_cast<float*>(wsb + lay.stat_text) : tvb_stat, wsb,
+                                 lay, split_total(p, ratio), tt ? nullptr : budgets, st);
+    if (e != cudaSuccess) return cuda_fail(e, "score launch");
+    if (score_launches(p) == 0) {   // no score kernel ran: split the (zero) statistic here
+        e = launch_budget(p, tvb_stat, split_total(p, ratio), budgets, status, st);
+        if (e != cudaSuccess) return cuda_fail(e, "budget launch");
+    }
+    e = launch_select_compact(p, scores, text_scores, budgets, modality, offsets, idx, k, v, k_out,
+                              v_out, retained_rows(p, ratio), status, st);
+    if (e != cudaSuccess) return cuda_fail(e, "select/compact launch");
+    return ok();
 }
 
 }  // namespace
@@ -379,64 +456,42 @@ int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* 
                 const float* w, double ratio, float* scores, float* tvb_stat, int32_t* budgets,
                 int64_t* offsets, int32_t* idx, uint16_t* k_out, uint16_t* v_out,
                 void* workspace, void* stream) {
+    return evict_impl(desc, q_text, k, v, modality, text_pos, w, ratio, false, nullptr, scores,
+                      tvb_stat, budgets, offsets, idx, k_out, v_out, workspace, stream);
+}
+
+int tgvkv_evict_with_stats(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* k,
+                           const uint16_t* v, const uint8_t* modality, const int32_t* text_pos,
+                           const float* w, double ratio, const float* row_stats, float* scores,
+                           float* tvb_stat, int32_t* budgets, int64_t* offsets, int32_t* idx,
+                           uint16_t* k_out, uint16_t* v_out, void* workspace, void* stream) {
+    return evict_impl(desc, q_text, k, v, modality, text_pos, w, ratio, true, row_stats, scores,
+                      tvb_stat, budgets, offsets, idx, k_out, v_out, workspace, stream);
+}
+
+int tgvkv_prefill(const tgvkv_desc* desc, const uint16_t* q, const uint16_t* k, const uint16_t* v,
+                  const uint8_t* modality, const int32_t* text_pos, uint16_t* o, uint16_t* q_text,
+                  float* row_stats, void* workspace, void* stream) {
     Problem p{};
     int rc = make_problem(desc, &p);
     if (rc) return rc;
-    if ((rc = check_ratio(ratio))) return rc;
-    rc = check_score_args(p, q_text, k, modality, text_pos, w, scores, tvb_stat, workspace,
-                          !p.weights_eq7);
-    if (rc) return rc;
+    if ((long long)p.L * p.H_q * p.N >= (1LL << 31))
+        return fail(TGVKV_ERR_UNSUPPORTED, "q holds 2^31 rows or more");
+    REQUIRE_PTR(q, "q", true);
+    REQUIRE_PTR(k, "k", true);
     REQUIRE_PTR(v, "v", true);
-    REQUIRE_PTR(budgets, "budgets", false);
-    REQUIRE_PTR(offsets, "offsets", false);
-    REQUIRE_PTR(idx, "idx", false);
-    REQUIRE_PTR(k_out, "k_out", true);
-    REQUIRE_PTR(v_out, "v_out", true);
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    REQUIRE_PTR(modality, "modality", false);
+    REQUIRE_PTR(o, "o", true);
+    if (p.n_win > 0) {
+        REQUIRE_PTR(text_pos, "text_pos", false);
+        REQUIRE_PTR(q_text, "q_text", true);
+        REQUIRE_PTR(row_stats, "row_stats", false);
+    }
+    REQUIRE_PTR(workspace, "workspace", true);
     const WsLayout lay = layout_of(p);
-    uint32_t* status = status_of(workspace, lay);
-    char* wsb = static_cast<char*>(workspace);
-    float* text_scores = nullptr;
-    if (needs_text_pass(p)) {
-        // Eq. 9 text scores (and Eq. 7 weights) into the workspace first
-        text_scores = reinterpret_cast<float*>(wsb + lay.text_scores);
-        float* wts = p.weights_eq7 ? reinterpret_cast<float*>(wsb + lay.weights) : nullptr;
-        // with TT budgeting the text pass's statistic (the text-text mass) is the one
-        // split, by that pass's last CTA
-        const bool tt = p.budget_stat == TGVKV_STAT_TT;
-        rc = do_text_scores(p, q_text, k, modality, text_pos, text_scores, p.n_win > 0 ? wts : nullptr,
-                            tt ? tvb_stat : reinterpret_cast<float*>(wsb + lay.stat_text), workspace, st,
-                            tt ? split_total(p, ratio) : -1, tt ? budgets : nullptr,
-                            reinterpret_cast<float*>(wsb + lay.row_stats));
-        if (rc) return rc;
-    }
-    Problem ps = p;
-    if (needs_text_pass(p)) {
-        // the vision pass takes the rows' (m, Z, vision mass) from the text-key
-        // pass instead of a pass A of its own
-        ps.row_stats = reinterpret_cast<float*>(wsb + lay.row_stats);
-        ps.stats_given = 1;
-    }
-    const float* w_used = w;
-    if (p.weights_eq7) {
-        w_used = reinterpret_cast<const float*>(wsb + lay.weights);
-        ps.w_stride = p.n_win;
-    }
-    // the score kernel's last CTA also derives the layer budgets (TV or uniform;
-    // with TT budgeting the text pass did, and the TV statistic goes to scratch)
-    const bool tt = p.budget_stat == TGVKV_STAT_TT;
-    cudaError_t e = launch_score(ps, q_text, k, modality, text_pos, w_used, scores,
-                                 tt ? reinterpret_cast<float*>(wsb + lay.stat_text) : tvb_stat, wsb,
-                                 lay, split_total(p, ratio), tt ? nullptr : budgets, st);
-    if (e != cudaSuccess) return cuda_fail(e, "score launch");
-    if (score_launches(p) == 0) {   // no score kernel ran: split the (zero) statistic here
-        e = launch_budget(p, tvb_stat, split_total(p, ratio), budgets, status, st);
-        if (e != cudaSuccess) return cuda_fail(e, "budget launch");
-    }
-    e = launch_select_compact(p, scores, text_scores, budgets, modality, offsets, idx, k, v, k_out,
-                              v_out, retained_rows(p, ratio), status, st);
-    if (e != cudaSuccess) return cuda_fail(e, "select/compact launch");
-    return ok();
+    cudaError_t e = launch_prefill(p, q, k, v, modality, text_pos, o, q_text, row_stats,
+                                   status_of(workspace, lay), static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ok() : cuda_fail(e, "prefill launch");
 }
 
 int tgvkv_decode(const tgvkv_desc* desc, const uint16_t* q, const uint16_t* k_rows,

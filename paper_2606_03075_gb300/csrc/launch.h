@@ -3,6 +3,7 @@
 // C-ABI layer.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -54,6 +55,18 @@ int decode_launches(const Problem& p);
 // Kernels launch_score / launch_select_compact launch for p.
 int score_launches(const Problem& p);
 int select_compact_launches(const Problem& p);
+
+// Causal prefill attention over every token (prefill.cu), which also writes
+// the eviction step's query rows (q_text) and their (m, Z, vision mass).
+cudaError_t launch_prefill(const Problem& p, const uint16_t* q, const uint16_t* k,
+                           const uint16_t* v, const uint8_t* modality, const int32_t* text_pos,
+                           uint16_t* o, uint16_t* q_text, float* row_stats, uint32_t* status,
+                           cudaStream_t stream);
+
+// TMA map of a bf16 [rows][d] tensor with boxes of 64 x box_rows, 128-byte
+// swizzle (score_tc.cu), and the SM count of the current device.
+bool make_tile_map(CUtensorMap* map, const void* base, uint64_t rows, int d, uint32_t box_rows);
+int device_sm_count();
 
 cudaError_t launch_compact(const Problem& p, const uint16_t* k, const uint16_t* v,
                            const int64_t* offsets, const int32_t* idx, uint16_t* k_out,

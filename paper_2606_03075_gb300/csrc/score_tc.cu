@@ -1187,6 +1187,12 @@ cudaError_t launch_tc(const Problem& p, const uint16_t* q, const uint16_t* k,
 
 }  // namespace
 
+bool make_tile_map(CUtensorMap* map, const void* base, uint64_t rows, int d, uint32_t box_rows) {
+    return make_map(map, base, rows, d, box_rows);
+}
+
+int device_sm_count() { return sm_count(); }
+
 int score_launches(const Problem& p) { return p.R == 0 ? 0 : 1; }
 
 cudaError_t launch_score(const Problem& p, const uint16_t* q, const uint16_t* k,

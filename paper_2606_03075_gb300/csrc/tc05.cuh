@@ -125,6 +125,35 @@ __device__ __forceinline__ void tmem_wait_ld() {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+// Store 32 consecutive 32-bit columns of this thread's TMEM lane (warp-wide).
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const float (&v)[32]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+        "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+        "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
+        "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
+        "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
+        "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+        "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+        "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])),
+        "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])),
+        "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])),
+        "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])),
+        "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])),
+        "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31]))
+        : "memory");
+}
+__device__ __forceinline__ void tmem_wait_st() {
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// Make this thread's ordinary shared-memory stores visible to the async proxy
+// (the tensor cores read MMA operands through it).
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 // ---- UMMA descriptors -----------------------------------------------------
 // Shared-memory matrix descriptor for a K-major operand stored in the 128-byte
 // swizzled layout that TMA writes (8-row x 128-byte atoms, 1024 bytes apart).
@@ -138,6 +167,20 @@ __device__ __forceinline__ uint64_t sdesc_k_sw128(uint32_t saddr) {
     return d;
 }
 
+// Descriptor of an MN-major operand in the same 128-byte swizzled layout: rows
+// of 64 MN elements (128 bytes) along K, 8-row atoms 1024 bytes apart along K,
+// and the next 64 MN elements `mn_stride` bytes further (a V tile as TMA
+// writes it: key rows of 64 dims, one box per 64 dims).
+__device__ __forceinline__ uint64_t sdesc_mn_sw128(uint32_t saddr, uint32_t mn_stride) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);       // start address, 16-byte units
+    d |= (uint64_t)((mn_stride >> 4) & 0x3FFFu) << 16;   // leading byte offset: next 64 MN elements
+    d |= (uint64_t)(1024u >> 4) << 32;               // stride byte offset: next 8 K rows
+    d |= (uint64_t)1u << 46;                         // descriptor version
+    d |= (uint64_t)2u << 61;                         // swizzle: 128 B
+    return d;
+}
+
 // Instruction descriptor, kind::f16: bf16 x bf16 -> fp32, both K-major.
 __host__ __device__ constexpr uint32_t idesc_bf16(int m, int n) {
     return (1u << 4)                          // D format: f32
@@ -145,6 +188,11 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int m, int n) {
            | (1u << 10)                       // B format: bf16
            | ((uint32_t)(n >> 3) << 17)       // N / 8
            | ((uint32_t)(m >> 4) << 24);      // M / 16
+}
+
+// The same with the B operand MN-major (transposed).
+__host__ __device__ constexpr uint32_t idesc_bf16_bmn(int m, int n) {
+    return idesc_bf16(m, n) | (1u << 16);
 }
 
 // D[tmem] (+)= A[smem] * B[smem]^T, issued by one thread.

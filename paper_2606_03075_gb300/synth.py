@@ -33,7 +33,7 @@ from dataclasses import dataclass, field
 
 import numpy as np
 
-_TAG_Q, _TAG_K, _TAG_V, _TAG_W = 1, 2, 3, 4
+_TAG_Q, _TAG_K, _TAG_V, _TAG_W, _TAG_QALL = 1, 2, 3, 4, 5
 
 
 @dataclass(frozen=True)
@@ -180,6 +180,27 @@ def generate(wl: Workload, seed: int = 0) -> dict:
         q[l], k[l], v[l], w[l] = draw_layer(wl, seed, l)
     return dict(q=q, k=k, v=v, w=w, modality=wl.modality,
                 text_pos=wl.text_pos.astype(np.int32))
+
+
+def draw_prefill_queries(wl: Workload, seed: int, layer: int, q_rows: np.ndarray) -> np.ndarray:
+    """Queries of every token of one layer, [H_q, N, d] int16 bf16 bits: the
+    query-row positions (text_pos) hold q_rows, that layer's q of draw_layer;
+    every other position holds a fresh N(0, 1) draw."""
+    r = _rng(seed, _TAG_QALL, layer)
+    q = to_bf16_bits(r.standard_normal((wl.H_q, wl.N, wl.d), dtype=np.float32))
+    q[:, wl.text_pos] = q_rows
+    return q
+
+
+def generate_prefill(wl: Workload, seed: int = 0, inp: dict | None = None) -> dict:
+    """generate() plus q_all [L, H_q, N, d]: the queries of every token, whose
+    rows at the query positions are generate()'s q."""
+    inp = dict(inp if inp is not None else generate(wl, seed))
+    q_all = np.empty((wl.L, wl.H_q, wl.N, wl.d), np.int16)
+    for l in range(wl.L):
+        q_all[l] = draw_prefill_queries(wl, seed, l, inp["q"][l])
+    inp["q_all"] = q_all
+    return inp
 
 
 def custom(name, L, H_q, H_kv, d, segments, **kw) -> Workload:
