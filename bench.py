@@ -603,6 +603,91 @@ def main():
         decode["full_frac"] = decode["full_gbs"] / pk
         del comp
 
+    # ---- the prefill side: causal attention over every token that also keeps
+    # the query rows' (m, Z, vision mass), then the eviction that reads them
+    # instead of running its own pass over the row statistics
+    prefill = None
+    if not args.no_next_rows:
+        pinp = synth.generate_prefill(wl, seed=args.seed + rank, inp=inp)
+        kv_bytes = 2 * inp["k"].nbytes
+        n_q = max(2, math.ceil(2 * L2_BYTES / (pinp["q_all"].nbytes + kv_bytes)) + 1)
+        q_alls = [upload(pinp["q_all"], torch.bfloat16) for _ in range(n_q)]
+        del pinp
+        o_pf = torch.empty_like(q_alls[0])
+        qt_pf = torch.empty((wl.L, wl.H_q, wl.n_win, wl.d), dtype=torch.bfloat16, device=dev)
+        rs_pf = torch.empty((wl.L, wl.H_q, wl.n_win, 3), dtype=torch.float32, device=dev)
+        # the same attention without query rows: no statistics to keep
+        desc_plain = api.make_desc(wl.L, wl.H_q, wl.H_kv, wl.d, wl.N, wl.N_v, 0)
+        ws_plain = api.new_workspace(desc_plain, dev)
+        n_pf = max(3, min(args.steps, 50))
+
+        def time_calls(call, n):
+            for s in range(3):
+                call(s)
+            barrier()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            for s in range(n):
+                call(3 + s)
+            b.record(stream)
+            barrier()
+            return a.elapsed_time(b) / n      # ms per call
+
+        def prefill_call(dsc, wsp):
+            def call(s):
+                x = sets[s % n_sets]
+                api.tgvkv_prefill(dsc, q_alls[s % n_q], x["k"], x["v"], x["modality"],
+                                  x["text_pos"], o_pf, qt_pf, rs_pf, wsp, stream)
+            return call
+
+        t_pf = time_calls(prefill_call(desc, ws), n_pf)
+        t_pf_plain = time_calls(prefill_call(desc_plain, ws_plain), n_pf)
+
+        def evict_stats(s):
+            x = sets[s % n_sets]
+            api.tgvkv_evict_with_stats(desc, qt_pf, x["k"], x["v"], x["modality"], x["text_pos"],
+                                       x["w"], ratio, rs_pf, out, ws, stream)
+
+        n_ev = max(3, min(args.steps, 200))
+        t_ev_stats = time_calls(evict_stats, n_ev)
+        bits = api.tgvkv_status(ws, stream) | api.tgvkv_status(ws_plain, stream)
+        if bits != 0:
+            raise RuntimeError(f"device status bits 0x{bits:x} set in the prefill runs")
+        # causal attention FLOPs: QK^T and PV over every visible (row, key) pair
+        pairs = wl.N * (wl.N + 1) // 2
+        flops = 4.0 * wl.d * wl.H_q * wl.L * pairs
+        peaks = measured_peaks()[0]
+        peak_tf = float(peaks.get("bf16_tflops", 0.0)) or None
+        tf = flops / (t_pf * 1e-3) / 1e12
+        prefill = {
+            "what": "causal prefill attention of every token (all layers) that also keeps the "
+                    "eviction rows' statistics; then tgvkv_evict_with_stats",
+            "prefill_ms": t_pf, "prefill_plain_ms": t_pf_plain,
+            "stats_overhead_frac": t_pf / t_pf_plain - 1.0,
+            "flops_per_launch": flops, "tflops": tf,
+            "frac_of_measured_bf16": tf / peak_tf if peak_tf else None,
+            "evict_with_stats_us_per_layer": t_ev_stats * 1e3 / wl.L,
+            "evict_us_per_layer": us_per_layer,
+            "evict_saving_frac": 1.0 - (t_ev_stats * 1e3 / wl.L) / us_per_layer,
+            "steps": n_pf}
+        # context only: the library attention (PyTorch SDPA) on the same tensors
+        try:
+            import torch.nn.functional as F
+            kq = sets[0]["k"].view(wl.L, wl.H_kv, wl.N, wl.d)
+            vq = sets[0]["v"].view(wl.L, wl.H_kv, wl.N, wl.d)
+
+            def sdpa(s):
+                F.scaled_dot_product_attention(q_alls[s % n_q], kq, vq, is_causal=True,
+                                               enable_gqa=wl.H_q != wl.H_kv)
+
+            t_sdpa = time_calls(sdpa, n_pf)
+            prefill["sdpa_ms"] = t_sdpa
+            prefill["sdpa_tflops"] = flops / (t_sdpa * 1e-3) / 1e12
+        except Exception as exc:   # noqa: BLE001 - context figure only
+            prefill["sdpa_ms"] = None
+            prefill["sdpa_error"] = str(exc)[:200]
+        del q_alls, o_pf
+
     # ---- end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
@@ -710,6 +795,7 @@ def main():
             "stage_ms": stage_ms,
             "next_rows": next_rows,
             "decode": decode,
+            "prefill": prefill,
             "fused_tail_ms": statistics.mean(step_ms) - stage_ms["score"],
             "step_ms_median": statistics.median(step_ms),
             "wall_s_timed_region": t_wall,

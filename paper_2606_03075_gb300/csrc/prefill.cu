@@ -30,10 +30,12 @@
 // 6): the prefill already streams every key of those rows.
 //
 // Roles: warp 0 issues the TMA loads, warp 1 the MMAs (and owns the TMEM),
-// warps 2-5 run the softmax, one per TMEM lane quarter.  Every wait is bounded
+// warps 2-5 run the softmax, one per TMEM lane quarter, warp 6 copies the
+// query rows to q_text.  Every wait is bounded
 // (about 1 s of SM cycles); a timeout sets TGVKV_STATUS_TIMEOUT and the CTA
 // unwinds after its copies and MMAs have finished.
 #include <cuda_bf16.h>
+#include <limits.h>
 #include <math.h>
 
 #include "common.cuh"
@@ -47,7 +49,8 @@ constexpr int PM = 128;                 // query rows per tile = TMEM lanes
 constexpr int PN = 128;                 // keys per K / V tile
 constexpr int PST = 4;                  // ring stages
 constexpr int P_NSW = 4;                // softmax warps
-constexpr int P_THREADS = (2 + P_NSW) * 32;
+constexpr int COPY_WARP = 2 + P_NSW;      // copies the query rows to q_text
+constexpr int P_THREADS = (3 + P_NSW) * 32;
 constexpr int P_TMEM_COLS = 512;        // S buffers at columns 0 and 128, O at 256
 constexpr uint32_t O_COL = 256;
 constexpr float kRescaleLog2 = 8.f;     // a stale reference maximum may trail by 2^8
@@ -63,6 +66,7 @@ struct FSmem {
     uint64_t p_full, o_done, mma_done;
     uint32_t tmem_base;
     int abort_flag, never;
+    int wtile[kMaxN / PM + 1];          // first query row at or after position 128 t
 };
 
 struct PItem {
@@ -119,32 +123,51 @@ __device__ __forceinline__ void qk_block(uint32_t d_tmem, uint64_t qdesc, uint64
     }
 }
 
-// One row of a score tile: P = 2^(x sl2 - m) for the keys c <= lim, packed in
-// bf16 pairs; returns the fp32 sum and adds the vision keys' part to vs when
-// want_v (vision bits of the 128 keys in vw).
-template <bool MASKED>
-__device__ __forceinline__ float exp_row(const float (&x)[PN], float sl2, float m, int lim,
-                                         bool want_v, const uint32_t (&vw)[4], uint32_t (&pk)[PN / 2],
+// One row of a score tile: P = 2^(x sl2 - m) for its 128 keys (a masked key
+// holds x = -inf, so P = 0 there), packed in bf16 pairs; returns the fp32 sum.
+// VISION: also adds the part over the vision keys (bits in vw, the same for
+// every lane of the warp) to vs, per 32-key word: the word's sum when it is all
+// vision, nothing when it is all text, key by key only for a mixed word.
+template <bool VISION>
+__device__ __forceinline__ float exp_row(const float (&x)[PN], float sl2, float m,
+                                         const uint32_t (&vw)[4], uint32_t (&pk)[PN / 2],
                                          float& vs) {
     const float2 s2 = make_float2(sl2, sl2), n2 = make_float2(-m, -m);
-    float2 za = make_float2(0.f, 0.f), va = za;
+    float z = 0.f;
 #pragma unroll
-    for (int c = 0; c < PN; c += 2) {
-        const float2 t = fma2(make_float2(x[c], x[c + 1]), s2, n2);
-        float e0 = fast_exp2(t.x), e1 = fast_exp2(t.y);
-        if (MASKED) {
-            if (c > lim) e0 = 0.f;
-            if (c + 1 > lim) e1 = 0.f;
+    for (int w = 0; w < PN / 32; ++w) {
+        float e[32];
+        float2 za = make_float2(0.f, 0.f), zb = za;
+#pragma unroll
+        for (int c = 0; c < 32; c += 4) {
+            const float2 t0 = fma2(make_float2(x[32 * w + c], x[32 * w + c + 1]), s2, n2);
+            const float2 t1 = fma2(make_float2(x[32 * w + c + 2], x[32 * w + c + 3]), s2, n2);
+            e[c] = fast_exp2(t0.x);
+            e[c + 1] = fast_exp2(t0.y);
+            e[c + 2] = fast_exp2(t1.x);
+            e[c + 3] = fast_exp2(t1.y);
+            pk[16 * w + c / 2] = pack_bf16(e[c], e[c + 1]);
+            pk[16 * w + c / 2 + 1] = pack_bf16(e[c + 2], e[c + 3]);
+            za = add2(za, make_float2(e[c], e[c + 1]));
+            zb = add2(zb, make_float2(e[c + 2], e[c + 3]));
         }
-        pk[c >> 1] = pack_bf16(e0, e1);
-        za = add2(za, make_float2(e0, e1));
-        if (want_v) {
-            const uint32_t w = vw[c >> 5];
-            va = add2(va, make_float2((w >> (c & 31)) & 1u ? e0 : 0.f, (w >> ((c + 1) & 31)) & 1u ? e1 : 0.f));
+        const float zw = (za.x + za.y) + (zb.x + zb.y);
+        z += zw;
+        if (VISION) {
+            const uint32_t bits = vw[w];
+            if (bits == ~0u) {
+                vs += zw;
+            } else if (bits != 0u) {
+                float2 va = make_float2(0.f, 0.f);
+#pragma unroll
+                for (int c = 0; c < 32; c += 2)
+                    va = add2(va, make_float2((bits >> c) & 1u ? e[c] : 0.f,
+                                              (bits >> (c + 1)) & 1u ? e[c + 1] : 0.f));
+                vs += va.x + va.y;
+            }
         }
     }
-    vs += va.x + va.y;
-    return za.x + za.y;
+    return z;
 }
 
 // Three-input maximum (PTX max.f32 with three sources).
@@ -154,20 +177,12 @@ __device__ __forceinline__ float fmax3f(float a, float b, float c) {
     return r;
 }
 
-template <bool MASKED>
-__device__ __forceinline__ float row_max(const float (&x)[PN], int lim) {
+__device__ __forceinline__ float row_max(const float (&x)[PN]) {
     float a = -INFINITY, b = -INFINITY;
 #pragma unroll
     for (int c = 0; c < PN; c += 4) {
-        if (MASKED) {
-            if (c <= lim) a = fmaxf(a, x[c]);
-            if (c + 1 <= lim) b = fmaxf(b, x[c + 1]);
-            if (c + 2 <= lim) a = fmaxf(a, x[c + 2]);
-            if (c + 3 <= lim) b = fmaxf(b, x[c + 3]);
-        } else {
-            a = fmax3f(a, x[c], x[c + 1]);
-            b = fmax3f(b, x[c + 2], x[c + 3]);
-        }
+        a = fmax3f(a, x[c], x[c + 1]);
+        b = fmax3f(b, x[c + 2], x[c + 3]);
     }
     return fmaxf(a, b);
 }
@@ -215,6 +230,34 @@ __global__ void __launch_bounds__(P_THREADS, 1)
     if (warp == 1) {
         tc::tmem_alloc(&s.tmem_base, P_TMEM_COLS);
         tc::tmem_relinquish();
+    }
+    // the query rows of each row tile t: indices wtile[t] .. wtile[t + 1] of
+    // text_pos (positions ascend), as the first row at or after position 128 t
+    for (int t = tid; t <= n_qt; t += P_THREADS) s.wtile[t] = p.n_win;
+    __syncthreads();
+    for (int i = tid; i < p.n_win; i += P_THREADS) {
+        const int pi = __ldg(text_pos + i);
+        if (pi >= 0 && pi < p.N) atomicMin(&s.wtile[pi / PM], i);
+    }
+    __syncthreads();
+    if (warp == 0) {
+        // suffix minimum over the tiles: per lane over a chunk, then across lanes
+        const int per = (n_qt + 1 + 31) / 32;
+        const int lo = lane * per, hi = lo + per < n_qt + 1 ? lo + per : n_qt + 1;
+        int run = INT_MAX;
+        for (int x = hi - 1; x >= lo; --x) {
+            run = min(run, s.wtile[x]);
+            s.wtile[x] = run;
+        }
+        int incl = run;                      // minimum over this lane's chunk and all later ones
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_down_sync(~0u, incl, o);
+            if (lane + o < 32) incl = min(incl, y);
+        }
+        int later = __shfl_down_sync(~0u, incl, 1);
+        if (lane == 31) later = INT_MAX;
+        for (int x = lo; x < hi; ++x) s.wtile[x] = min(s.wtile[x], later);
     }
     tc::fence_before_sync();
     __syncthreads();
@@ -340,7 +383,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
     }
 
     // ------------------------------------------------------------ softmax
-    if (warp >= 2) {
+    if (warp >= 2 && warp < COPY_WARP) {
         const int quarter = warp & 3;
         const int r = quarter * 32 + lane;                   // this thread's row = TMEM lane
         const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16);
@@ -352,32 +395,44 @@ __global__ void __launch_bounds__(P_THREADS, 1)
             const int nk = itm.t + 1;
             const int pos = itm.t * PM + r;
             const bool valid = pos < p.N;
-            // query row of the eviction step at this position (text_pos ascends)
+            // query row of the eviction step at this position: the tile's rows
+            // are text_pos[ws .. we); those on this warp's 32 positions set bits
+            const int base = itm.t * PM + quarter * 32;
+            const int ws = s.wtile[itm.t], we = s.wtile[itm.t + 1];
             int wi = -1;
-            if (valid && p.n_win > 0) {
-                int lo = 0, hi = p.n_win - 1;
-                while (lo <= hi) {
-                    const int mid = (lo + hi) >> 1;
-                    const int tp = __ldg(text_pos + mid);
-                    if (tp == pos) {
-                        wi = mid;
-                        break;
-                    }
-                    if (tp < pos) lo = mid + 1;
-                    else hi = mid - 1;
+            if (we > ws) {
+                uint32_t hit = 0u;
+                int below = 0;
+                for (int k0 = ws; k0 < we; k0 += 32) {
+                    const int e = k0 + lane;
+                    const int pe = e < we ? __ldg(text_pos + e) : INT_MAX;
+                    below += __popc(__ballot_sync(~0u, pe < base));
+                    const bool in = pe >= base && pe - base < 32;
+                    hit |= __reduce_or_sync(~0u, in ? 1u << (pe - base) : 0u);
                 }
+                if (valid && ((hit >> lane) & 1u)) wi = ws + below + __popc(hit & ((1u << lane) - 1u));
             }
             const bool want_v = __any_sync(~0u, wi >= 0);
             float m = -INFINITY, lsum = 0.f, vsum = 0.f;
+            // modality bytes of key tile j (this lane's keys 32 w + lane), loaded one
+            // tile ahead and first used a tile later, so that the loads' latency
+            // hides behind a tile of work
+            int mod_next[4] = {0, 0, 0, 0};
+            auto load_modality = [&](int j) {
+#pragma unroll
+                for (int w = 0; w < 4; ++w) {
+                    const int key = j * PN + 32 * w + lane;
+                    mod_next[w] = key < p.N ? (int)__ldg(modality + key) : 0;
+                }
+            };
+            if (want_v) load_modality(0);
             for (int j = 0; j < nk; ++j) {
                 const int b = st & 1;
                 uint32_t vw[4] = {0u, 0u, 0u, 0u};
                 if (want_v) {
 #pragma unroll
-                    for (int w = 0; w < 4; ++w) {
-                        const int key = j * PN + 32 * w + lane;
-                        vw[w] = __ballot_sync(~0u, key < p.N && __ldg(modality + key) != 0);
-                    }
+                    for (int w = 0; w < 4; ++w) vw[w] = __ballot_sync(~0u, mod_next[w] != 0);
+                    if (j + 1 < nk) load_modality(j + 1);
                 }
                 if (!warp_wait_all(&s.s_full[b], (st >> 1) & 1, abort_flag)) {
                     ok = false;
@@ -399,10 +454,14 @@ __global__ void __launch_bounds__(P_THREADS, 1)
                 __syncwarp();
                 if (lane == 0) tc::mbar_arrive(&s.s_empty[b]);
 
-                // keys c <= lim are visible: all of them below the diagonal tile
-                const bool diag = j == itm.t;
-                const int lim = diag ? r : PN - 1;
-                const float m_tile = (diag ? row_max<true>(x, lim) : row_max<false>(x, lim)) * sl2;
+                // keys c <= r are visible in the diagonal tile, all of them below it;
+                // a masked logit becomes -inf, so that 2^(x sl2 - m) is 0 there
+                if (j == itm.t) {
+#pragma unroll
+                    for (int c = 0; c < PN; ++c)
+                        if (c > r) x[c] = -INFINITY;
+                }
+                const float m_tile = row_max(x) * sl2;
                 float alpha = 1.f;
                 if (m_tile > m + kRescaleLog2) {   // also the first tile (m = -inf)
                     alpha = fast_exp2(m - m_tile);
@@ -411,9 +470,11 @@ __global__ void __launch_bounds__(P_THREADS, 1)
                     vsum *= alpha;
                 }
                 uint32_t pk[PN / 2];
-                const bool mine_v = wi >= 0;
-                lsum += diag ? exp_row<true>(x, sl2, m, lim, want_v && mine_v, vw, pk, vsum)
-                             : exp_row<false>(x, sl2, m, lim, want_v && mine_v, vw, pk, vsum);
+                // (lanes without a query row sum a vision mass that is never written)
+                if (want_v)
+                    lsum += exp_row<true>(x, sl2, m, vw, pk, vsum);
+                else
+                    lsum += exp_row<false>(x, sl2, m, vw, pk, vsum);
 
                 // PV_{j-1} has finished: the P buffer and O are free
                 if (j > 0) {
@@ -488,13 +549,29 @@ __global__ void __launch_bounds__(P_THREADS, 1)
                 row_stats[3 * qr] = m;
                 row_stats[3 * qr + 1] = lsum;
                 row_stats[3 * qr + 2] = vsum;
-                const uint4* src = reinterpret_cast<const uint4*>(q + ((size_t)itm.lhq * p.N + pos) * D);
-                uint4* dst = reinterpret_cast<uint4*>(q_text + qr * D);
-#pragma unroll
-                for (int c = 0; c < D / 8; ++c) dst[c] = __ldg(src + c);
             }
         }
         if (!ok) raise_status(status, TGVKV_STATUS_TIMEOUT);
+    }
+
+    // ------------------------------------------------------------ query-row copies
+    // q_text[l][h][r] = q[l][h][text_pos[r]], for the rows of this CTA's items,
+    // D / 8 lanes per row (16 bytes each); independent of the other roles
+    if (warp == COPY_WARP) {
+        constexpr int LPR = D / 8, RPI = 32 / LPR;
+        const int sub = lane / LPR, c = lane % LPR;
+        for (int i = blockIdx.x; i < n_items; i += gridDim.x) {
+            const PItem itm = prefill_item(p, n_qt, i);
+            const int ws = s.wtile[itm.t], we = s.wtile[itm.t + 1];
+            const size_t qrow = ((size_t)itm.l * p.H_q + itm.h) * p.n_win;
+#pragma unroll 4
+            for (int e = ws + sub; e < we; e += RPI) {
+                const int pos = __ldg(text_pos + e);
+                if (pos < 0 || pos >= p.N) continue;
+                const uint4 v4 = __ldg(reinterpret_cast<const uint4*>(q + ((size_t)itm.lhq * p.N + pos) * D) + c);
+                reinterpret_cast<uint4*>(q_text + (qrow + e) * D)[c] = v4;
+            }
+        }
     }
 
     // ------------------------------------------------------------ teardown
