@@ -181,3 +181,36 @@ def test_head_budget_options(lib):
     assert lib.tgvkv_evict_launches(ref(_desc(**base, head_budgets=2))) == -1
     big = dict(base, L=64, H_q=32, H_kv=32)            # 2048 heads
     assert lib.tgvkv_evict_launches(ref(_desc(**big, head_budgets=1))) == -1
+
+
+def test_prefill_and_given_statistics_validation(lib):
+    """tgvkv_prefill / tgvkv_evict_with_stats reject bad arguments on the host:
+    null or misaligned buffers, an unsupported head size, TT budgets with given
+    statistics (they need each row's text mass)."""
+    P = ctypes.c_void_p
+    fake = P(0x1000)
+    odd = P(0x1008)
+    d = _desc()
+    ref = ctypes.byref
+
+    def prefill(desc, q=fake, o=fake, q_text=fake, stats=fake, text_pos=fake):
+        return lib.tgvkv_prefill(desc, q, fake, fake, fake, text_pos, o, q_text, stats, fake, None)
+
+    assert prefill(None) == 1
+    assert prefill(ref(_desc(d=96))) == 2
+    assert prefill(ref(d), q=P(0)) == 1
+    assert prefill(ref(d), o=odd) == 1
+    assert prefill(ref(d), q_text=odd) == 1
+    assert prefill(ref(d), stats=P(0)) == 1
+    assert prefill(ref(d), text_pos=P(0)) == 1
+    assert b"text_pos" in lib.tgvkv_last_error()
+
+    def evict_stats(desc, stats=fake, ratio=0.1):
+        return lib.tgvkv_evict_with_stats(desc, fake, fake, fake, fake, fake, fake, ratio, stats,
+                                          fake, fake, fake, fake, fake, fake, fake, fake, None)
+
+    assert evict_stats(ref(d), stats=P(0)) == 1
+    assert b"row_stats" in lib.tgvkv_last_error()
+    assert evict_stats(ref(d), ratio=1.5) == 1
+    assert evict_stats(ref(_desc(budget_stat=1))) == 2       # TGVKV_STAT_TT
+    assert b"TT" in lib.tgvkv_last_error()
