@@ -268,3 +268,36 @@ def test_full_size_prefill_then_evict(api, name, ratio, layers):
     assert g["budgets"].tolist() == oracle.tvb_budgets(g["stat"], total, wl.N_v)
     P.check_selection_and_compaction(wl, inp, g, layers, ref_scores=ref_s)
     assert g["offsets"][-1] == wl.H_kv * (wl.L * wl.N_t + total)
+
+
+def test_prefill_without_query_rows(api):
+    """The plain causal attention (no query rows: no statistics, no q_text)."""
+    wl = CASES["gqa_d64"]
+    inp = synth.generate_prefill(wl, seed=6)
+    desc = api.make_desc(wl.L, wl.H_q, wl.H_kv, wl.d, wl.N, wl.N_v, 0)
+    dev = P.device_inputs(inp)
+    q_all = _bf16(inp["q_all"])
+    o = torch.empty_like(q_all)
+    ws = api.new_workspace(desc)
+    api.tgvkv_prefill(desc, q_all, dev["k"], dev["v"], dev["modality"], None, o, None, None, ws)
+    assert api.tgvkv_status(ws) == 0
+    o_ref, bound = oracle.prefill_attention(oracle.widen_bf16(inp["q_all"]),
+                                            oracle.widen_bf16(inp["k"]),
+                                            oracle.widen_bf16(inp["v"]), 1.0 / math.sqrt(wl.d),
+                                            wl.H_kv)
+    err = np.abs(oracle.widen_bf16(o.view(torch.int16).cpu().numpy()) - o_ref)
+    assert np.all(err <= 2.0 ** -7 * bound + 1e-6), (err - 2.0 ** -7 * bound).max()
+
+
+def test_prefill_repeated_calls_bit_identical(api):
+    """Back-to-back launches on one workspace give the same bits (the schedule
+    does not change any sum)."""
+    wl = CASES["gqa_video"]
+    inp = synth.generate_prefill(wl, seed=7)
+    dev = P.device_inputs(inp)
+    first = [t.clone() for t in _run_prefill(api, wl, inp, dev)]
+    for _ in range(5):
+        again = _run_prefill(api, wl, inp, dev)
+        for a, b in zip(first, again):
+            assert torch.equal(a.view(torch.int16) if a.dtype == torch.bfloat16 else a,
+                               b.view(torch.int16) if b.dtype == torch.bfloat16 else b)
