@@ -158,9 +158,6 @@ long long split_total(const Problem& p, double ratio) {
     return p.head_budgets ? (long long)p.H_kv * budget_total(p, ratio) : budget_total(p, ratio);
 }
 
-// The cap of one layer's budget in the split.
-int budget_cap(const Problem& p) { return p.basis == TGVKV_BASIS_ALL ? p.N : p.N_v; }
-
 // Sink positions (at most N).
 int n_sinks(const Problem& p) {
     const int both = p.keep_first + p.keep_last;
