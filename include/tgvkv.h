@@ -319,6 +319,14 @@ int tgvkv_workspace_init(const tgvkv_desc* desc, void* workspace, void* stream);
  * value if the synchronisation itself failed. */
 int tgvkv_status(void* workspace, void* stream);
 
+/* Self-test of the failure detection (no counterpart in the paper).  Launches
+ * one CTA that waits, with the same bounded wait every kernel of the library
+ * uses, on an mbarrier that nothing arrives at.  The wait gives up after its
+ * limit (2e9 SM cycles, about 1 s) and the kernel sets TGVKV_STATUS_TIMEOUT in
+ * the status word of `workspace`, which tgvkv_status then returns; nothing
+ * faults and the context stays usable.  Returns TGVKV_OK once launched. */
+int tgvkv_check_wait_timeout(void* workspace, void* stream);
+
 /* Message of the last error returned on the calling thread ("" if none). */
 const char* tgvkv_last_error(void);
 

@@ -63,6 +63,7 @@ SIGNATURES = {
     "tgvkv_decode": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                              c_void_p]),
     "tgvkv_decode_launches": (c_int, [_P]),
+    "tgvkv_check_wait_timeout": (c_int, [c_void_p, c_void_p]),
     "tgvkv_last_error": (c_char_p, []),
     "tgvkv_score_noalloc": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                     c_void_p, c_void_p, c_void_p]),

@@ -305,6 +305,13 @@ def tgvkv_prefill(desc, q, k, v, modality, text_pos, o, q_text, row_stats, ws, s
         _stream(stream)), "tgvkv_prefill")
 
 
+def tgvkv_check_wait_timeout(ws: torch.Tensor, stream=None):
+    """Launch the failure-detection self-test: a bounded wait that runs out and
+    sets TGVKV_STATUS_TIMEOUT in the workspace's status word."""
+    _check(_lib.load().tgvkv_check_wait_timeout(_ptr(ws, (torch.uint8,), 4, "workspace"),
+                                                _stream(stream)), "tgvkv_check_wait_timeout")
+
+
 def tgvkv_status(ws: torch.Tensor, stream=None) -> int:
     """Synchronise the stream, return and clear the device status bits."""
     rc = _lib.load().tgvkv_status(_ptr(ws, (torch.uint8,), 4, "workspace"), _stream(stream))

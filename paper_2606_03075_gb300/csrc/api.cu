@@ -510,6 +510,14 @@ int tgvkv_decode(const tgvkv_desc* desc, const uint16_t* q, const uint16_t* k_ro
     return e == cudaSuccess ? ok() : cuda_fail(e, "decode launch");
 }
 
+int tgvkv_check_wait_timeout(void* workspace, void* stream) {
+    REQUIRE_PTR(workspace, "workspace", true);
+    // the status word is the first word of every workspace layout
+    cudaError_t e = launch_wait_timeout(static_cast<uint32_t*>(workspace),
+                                        static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ok() : cuda_fail(e, "wait-timeout launch");
+}
+
 int tgvkv_decode_launches(const tgvkv_desc* desc) {
     Problem p{};
     if (make_problem(desc, &p) != TGVKV_OK) return -1;

@@ -68,6 +68,10 @@ cudaError_t launch_prefill(const Problem& p, const uint16_t* q, const uint16_t* 
 bool make_tile_map(CUtensorMap* map, const void* base, uint64_t rows, int d, uint32_t box_rows);
 int device_sm_count();
 
+// One CTA that waits, with the library's bounded wait, on an mbarrier nothing
+// arrives at; the wait runs out and sets TGVKV_STATUS_TIMEOUT (selftest.cu).
+cudaError_t launch_wait_timeout(uint32_t* status, cudaStream_t stream);
+
 cudaError_t launch_compact(const Problem& p, const uint16_t* k, const uint16_t* v,
                            const int64_t* offsets, const int32_t* idx, uint16_t* k_out,
                            uint16_t* v_out, long long capacity_rows, uint32_t* status,
