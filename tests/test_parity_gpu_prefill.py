@@ -301,3 +301,40 @@ def test_prefill_repeated_calls_bit_identical(api):
         for a, b in zip(first, again):
             assert torch.equal(a.view(torch.int16) if a.dtype == torch.bfloat16 else a,
                                b.view(torch.int16) if b.dtype == torch.bfloat16 else b)
+
+
+FULL_LONG = [("next", 0.05, 31, 640), ("video", 0.05, 27, 512)]
+
+
+@pytest.mark.parametrize("name,ratio,layer,n_prefix", FULL_LONG)
+def test_full_size_long_prefill_then_evict(api, name, ratio, layer, n_prefix):
+    """The long workloads at full size: o of one layer's first n_prefix rows
+    (causal rows below n_prefix see only the first n_prefix keys, so the oracle
+    on the truncated sequence is exact for them), the query rows' statistics
+    over all keys, then the eviction with those statistics on that layer."""
+    wl = synth.WORKLOADS[name]
+    inp = synth.generate_prefill(wl, seed=0)
+    dev = P.device_inputs(inp)
+    o, q_text, stats = _run_prefill(api, wl, inp, dev)
+    scale = 1.0 / math.sqrt(wl.d)
+    q1 = oracle.widen_bf16(inp["q_all"][layer:layer + 1])
+    k1 = oracle.widen_bf16(inp["k"][layer:layer + 1])
+    v1 = oracle.widen_bf16(inp["v"][layer:layer + 1])
+    o_ref, bound = oracle.prefill_attention(q1[:, :, :n_prefix], k1[:, :, :n_prefix],
+                                            v1[:, :, :n_prefix], scale, wl.H_kv)
+    o_gpu = oracle.widen_bf16(o.view(torch.int16)[layer:layer + 1, :, :n_prefix].cpu().numpy())
+    assert np.all(np.abs(o_gpu - o_ref) <= 2.0 ** -7 * bound + 1e-6)
+    np.testing.assert_array_equal(q_text.view(torch.int16)[layer].cpu().numpy(),
+                                  inp["q"][layer])
+    lse2, vis = oracle.row_statistics(q1, k1, inp["modality"], inp["text_pos"], scale, wl.H_kv)
+    st = stats[layer:layer + 1].cpu().numpy().astype(np.float64)
+    assert np.all(np.abs(st[..., 0] + np.log2(st[..., 1]) - lse2) <= 1e-3)
+    P.assert_close(st[..., 2] / st[..., 1], vis, f"{name} vision share")
+    g = _run_evict_with_stats(api, wl, dev, q_text, stats, ratio)
+    assert g["status"] == 0
+    ref_s, ref_t = P.oracle_scores(wl, inp, [layer])
+    P.assert_close(g["scores"][[layer]], ref_s, f"{name} scores")
+    P.assert_close(g["stat"][[layer]], ref_t, f"{name} tvb_stat")
+    total = oracle.vision_budget_total(ratio, wl.N_v, wl.L)
+    assert g["budgets"].tolist() == oracle.tvb_budgets(g["stat"], total, wl.N_v)
+    P.check_selection_and_compaction(wl, inp, g, [layer], ref_scores=ref_s)
