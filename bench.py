@@ -97,6 +97,16 @@ def step_bytes(wl, ratio):
     return k_read + kv_written, rows
 
 
+def full_step_bytes(wl, ratio):
+    """All algorithmic bytes of one fused step: K read once, Q read, scores
+    written and read back, the kept K/V rows read and written, idx and offsets."""
+    _, rows = step_bytes(wl, ratio)
+    k = wl.L * wl.H_kv * wl.N * wl.d * 2
+    q = wl.L * wl.H_q * wl.n_win * wl.d * 2
+    scores = wl.L * wl.H_kv * wl.N_v * 4
+    return k + q + 2 * scores + 4 * rows * wl.d * 2 + 4 * rows + 8 * (wl.L * wl.H_kv + 1)
+
+
 def stage_bytes(wl, ratio):
     """Algorithmic bytes of each kernel launch (all layers)."""
     _, rows = step_bytes(wl, ratio)
@@ -766,6 +776,8 @@ def main():
     mufu["frac"] = mufu["achieved_G_per_s"] / mufu["peak_G_per_s"]
     sbytes, rows = step_bytes(wl, ratio)
     step_gbs = sbytes * args.steps * world / (region_ms * 1e-3) / 1e9
+    fbytes = full_step_bytes(wl, ratio)
+    full_gbs = fbytes * args.steps * world / (region_ms * 1e-3) / 1e9
 
     line = None
     if rank == 0:
@@ -785,7 +797,11 @@ def main():
             "hbm_step": {"bytes_per_step": sbytes, "bytes_per_layer": sbytes / wl.L,
                          "gbs": step_gbs, "peak": hbm_peak, "frac": step_gbs / hbm_peak,
                          "frac_nominal": step_gbs / NOMINAL_HBM_GBS,
-                         "definition": "K read once + compacted K/V written, per step"},
+                         "definition": "K read once + compacted K/V written, per step",
+                         "full_bytes_per_step": fbytes, "full_gbs": full_gbs,
+                         "full_frac": full_gbs / hbm_peak,
+                         "full_definition": "plus Q read, scores written and read, kept K/V "
+                                            "rows read, idx and offsets"},
             "roofline": {"bound": roof["bound"], "kernel": dom, "achieved": roof["achieved"],
                          "peak": roof["peak"], "unit": roof["unit"], "frac": roof["frac"],
                          "traffic": traffic, "bytes_per_launch": sb[dom],
