@@ -267,9 +267,10 @@ int tgvkv_prefill(const tgvkv_desc* desc, const uint16_t* q, const uint16_t* k,
 /* tgvkv_evict with the query rows' statistics given: row_stats as tgvkv_prefill
  * writes them (fp32 [L][H_q][n_win][3]).  The score passes then read each
  * row's (m, Z, vision mass) instead of streaming its keys a first time; all
- * other arguments and every result are those of tgvkv_evict.  Budgets by the
- * TT statistic need each row's text mass, which row_stats does not hold:
- * TGVKV_ERR_UNSUPPORTED. */
+ * other arguments and every result are those of tgvkv_evict.  Under TT
+ * budgeting the text-key pass keeps its own row statistics (its statistic is
+ * each row's text mass, which row_stats does not hold); the vision pass reads
+ * the given ones. */
 int tgvkv_evict_with_stats(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* k,
                            const uint16_t* v, const uint8_t* modality, const int32_t* text_pos,
                            const float* w, double ratio, const float* row_stats,

@@ -252,9 +252,6 @@ int evict_impl(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* k
     int rc = make_problem(desc, &p);
     if (rc) return rc;
     if ((rc = check_ratio(ratio))) return rc;
-    if (stats_given && p.budget_stat == TGVKV_STAT_TT)
-        return fail(TGVKV_ERR_UNSUPPORTED,
-                    "TT budgets need the rows' text mass, which the given statistics do not hold");
     if (stats_given && p.n_win > 0) REQUIRE_PTR(given_stats, "row_stats", false);
     // with no query rows (n_win = 0) no score pass runs and nothing is read
     float* stats = stats_given && p.n_win > 0 ? const_cast<float*>(given_stats) : nullptr;
@@ -280,12 +277,15 @@ int evict_impl(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* k
         // split, by that pass's last CTA
         const bool tt = p.budget_stat == TGVKV_STAT_TT;
         // the text-key pass computes the rows' (m, Z, vision mass) into the
-        // workspace, or reads the given ones
+        // workspace, or reads the given ones -- except under TT budgeting, whose
+        // statistic is each row's text mass, which the given statistics do not
+        // hold: then the text-key pass keeps its own row statistics
+        const bool text_reads = stats != nullptr && !tt;
         rc = do_text_scores(p, q_text, k, modality, text_pos, text_scores, p.n_win > 0 ? wts : nullptr,
                             tt ? tvb_stat : reinterpret_cast<float*>(wsb + lay.stat_text), workspace, st,
                             tt ? split_total(p, ratio) : -1, tt ? budgets : nullptr,
-                            stats ? stats : reinterpret_cast<float*>(wsb + lay.row_stats),
-                            stats != nullptr);
+                            text_reads ? stats : reinterpret_cast<float*>(wsb + lay.row_stats),
+                            text_reads);
         if (rc) return rc;
     }
     Problem ps = p;

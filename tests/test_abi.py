@@ -185,8 +185,7 @@ def test_head_budget_options(lib):
 
 def test_prefill_and_given_statistics_validation(lib):
     """tgvkv_prefill / tgvkv_evict_with_stats reject bad arguments on the host:
-    null or misaligned buffers, an unsupported head size, TT budgets with given
-    statistics (they need each row's text mass)."""
+    null or misaligned buffers, an unsupported head size, a bad ratio."""
     P = ctypes.c_void_p
     fake = P(0x1000)
     odd = P(0x1008)
@@ -212,5 +211,3 @@ def test_prefill_and_given_statistics_validation(lib):
     assert evict_stats(ref(d), stats=P(0)) == 1
     assert b"row_stats" in lib.tgvkv_last_error()
     assert evict_stats(ref(d), ratio=1.5) == 1
-    assert evict_stats(ref(_desc(budget_stat=1))) == 2       # TGVKV_STAT_TT
-    assert b"TT" in lib.tgvkv_last_error()

@@ -17,7 +17,7 @@ Tolerances, from the arithmetic of the kernel:
   * the eviction with the given statistics: the bar of the eviction tests --
     scores and statistic within 1e-3 of the oracle (2e-3 with Eq. 7 weights),
     budgets, retained sets and compacted rows exact given the GPU's statistic
-    and scores.
+    and scores; TT budgeting included.
 """
 import math
 
@@ -236,13 +236,26 @@ def test_evict_with_prefill_statistics_widened(api, name):
                     _kept_gap_rule(ref, b - len(sink_t), set(cand), (l, h))
 
 
-def test_evict_with_statistics_rejects_tt(api):
+def test_evict_with_statistics_tt_budgets(api):
+    """TT budgeting with given statistics: the text-key pass keeps its own row
+    statistics (the TT statistic is each row's text mass), the vision pass reads
+    the given ones; statistic, budgets, scores and sets against the oracle."""
     wl = CASES["mha_ragged"]
     inp = synth.generate_prefill(wl, seed=5)
     dev = P.device_inputs(inp)
     _, q_text, stats = _run_prefill(api, wl, inp, dev)
-    with pytest.raises(api.TgvkvError):
-        _run_evict_with_stats(api, wl, dev, q_text, stats, 0.1, stat="tt")
+    ratio = 0.1
+    g = _run_evict_with_stats(api, wl, dev, q_text, stats, ratio, stat="tt")
+    assert g["status"] == 0
+    ref = oracle.evict(inp["q"], inp["k"], inp["v"], inp["modality"], inp["text_pos"], inp["w"],
+                       ratio, wl.H_kv, budget_stat="tt")
+    P.assert_close(g["stat"], ref["stat"], "TT statistic")
+    P.assert_close(g["scores"], ref["scores"], "scores")
+    total = oracle.vision_budget_total(ratio, wl.N_v, wl.L)
+    assert g["budgets"].tolist() == oracle.tvb_budgets(g["stat"], total, wl.N_v)
+    P.check_selection_and_compaction(wl, inp, g, list(range(wl.L)),
+                                     ref_scores=ref["scores"] if np.array_equal(
+                                         g["budgets"], ref["budgets"]) else None)
 
 
 FULL = [("llava15", 0.05, (0, 31)), ("qwen25", 0.05, (13,))]
