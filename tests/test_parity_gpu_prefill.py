@@ -133,7 +133,8 @@ def _run_evict_with_stats(api, wl, dev, q_text, stats, ratio, **options):
     api.tgvkv_evict_with_stats(desc, q_text, dev["k"], dev["v"], dev["modality"], dev["text_pos"],
                                dev["w"], ratio, stats, out, ws)
     status = api.tgvkv_status(ws)
-    rows = api.tgvkv_retained_rows(desc, ratio)
+    rows = int(out.offsets[-1].item())
+    assert rows <= api.tgvkv_retained_rows(desc, ratio)
     return dict(scores=out.scores.cpu().numpy(), stat=out.tvb_stat.cpu().numpy(),
                 budgets=out.budgets.cpu().numpy().astype(np.int64),
                 offsets=out.offsets.cpu().numpy(),
@@ -351,3 +352,33 @@ def test_full_size_long_prefill_then_evict(api, name, ratio, layer, n_prefix):
     total = oracle.vision_budget_total(ratio, wl.N_v, wl.L)
     assert g["budgets"].tolist() == oracle.tvb_budgets(g["stat"], total, wl.N_v)
     P.check_selection_and_compaction(wl, inp, g, [layer], ref_scores=ref_s)
+
+
+@pytest.mark.parametrize("stat", ["tv", "uniform"])
+def test_evict_with_statistics_head_budgets(api, stat):
+    """Head-adaptive budgets with given statistics: the per-head TV masses come
+    from the prefill's rows; budgets, CSR, sets and rows exact given them."""
+    wl = CASES["gqa_video"]
+    inp = synth.generate_prefill(wl, seed=8)
+    dev = P.device_inputs(inp)
+    _, q_text, stats = _run_prefill(api, wl, inp, dev)
+    ratio = 0.2
+    g = _run_evict_with_stats(api, wl, dev, q_text, stats, ratio, stat=stat, head_budgets=True)
+    assert g["status"] == 0
+    L, H = wl.L, wl.H_kv
+    total = oracle.vision_budget_total(ratio, wl.N_v, L)
+    if stat == "tv":
+        q, k = oracle.widen_bf16(inp["q"]), oracle.widen_bf16(inp["k"])
+        ref = oracle.tv_statistic_per_head(q, k, inp["modality"], inp["text_pos"],
+                                           1.0 / math.sqrt(wl.d), H)
+        P.assert_close(g["stat"].reshape(L, H), ref, "per-head TV mass")
+    stat_used = g["stat"] if stat == "tv" else np.zeros(L * H)
+    budgets = np.asarray(oracle.tvb_budgets(stat_used, H * total, wl.N_v)).reshape(L, H)
+    np.testing.assert_array_equal(g["budgets"].reshape(L, H), budgets)
+    off, idx = oracle.tpr_select_general(g["scores"], None, budgets, inp["modality"],
+                                         vision_basis=True)
+    np.testing.assert_array_equal(g["offsets"], off)
+    np.testing.assert_array_equal(g["idx"], idx)
+    ko, vo = oracle.compact(inp["k"], inp["v"], off, idx)
+    np.testing.assert_array_equal(g["k_out"], ko)
+    np.testing.assert_array_equal(g["v_out"], vo)
