@@ -106,3 +106,42 @@ def test_two_cpu_ranks_match_the_unsharded_oracle():
         np.testing.assert_array_equal(p["k_out"], ref["k_out"][lo:hi])
         np.testing.assert_array_equal(p["v_out"], ref["v_out"][lo:hi])
     assert sum(int(p["l1"]) - int(p["l0"]) for p in parts) == WL.L
+
+
+def _rank_leaves(rank, world, port, outdir):
+    """Rank 1 leaves between steps, without joining the statistic's exchange;
+    rank 0's exchange must end with an error within the group's timeout
+    instead of waiting for it forever."""
+    import datetime
+    import time
+    dist.init_process_group("gloo", init_method=f"tcp://127.0.0.1:{port}", rank=rank,
+                            world_size=world, timeout=datetime.timedelta(seconds=10))
+    try:
+        if rank == 1:
+            open(os.path.join(outdir, "r1_left"), "w").close()
+            return
+        inp = synth.generate(WL, seed=7)
+        l0, l1 = shard.layer_range(WL.L, rank, world)
+        local = {k: torch.from_numpy(np.ascontiguousarray(inp[k][l0:l1])) for k in ("q", "k", "v", "w")}
+        local["modality"] = torch.from_numpy(inp["modality"])
+        local["text_pos"] = torch.from_numpy(inp["text_pos"].astype(np.int32))
+        t0 = time.time()
+        try:
+            shard.sharded_evict(_desc(WL), local, 0.2, rank, world, OracleBackend())
+            outcome = "completed"
+        except Exception as exc:      # the failed exchange surfaces as an error
+            outcome = f"error {time.time() - t0:.1f} {type(exc).__name__}"
+        with open(os.path.join(outdir, "r0.txt"), "w") as f:
+            f.write(outcome)
+    finally:
+        dist.destroy_process_group()
+
+
+def test_a_rank_that_leaves_fails_the_exchange_instead_of_hanging():
+    world = 2
+    with tempfile.TemporaryDirectory() as outdir:
+        mp.spawn(_rank_leaves, args=(world, _free_port(), outdir), nprocs=world, join=True)
+        assert os.path.exists(os.path.join(outdir, "r1_left"))
+        outcome = open(os.path.join(outdir, "r0.txt")).read().split()
+        assert outcome[0] == "error", outcome
+        assert float(outcome[1]) < 30.0
