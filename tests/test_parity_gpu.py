@@ -334,3 +334,51 @@ def test_layer_sharded_ranks_match_full_evict(api):
         np.testing.assert_array_equal(idx.cpu().numpy(), full["idx"][lo:hi])
         np.testing.assert_array_equal(ko.view(torch.int16).cpu().numpy(), full["k_out"][lo:hi])
         np.testing.assert_array_equal(vo.view(torch.int16).cpu().numpy(), full["v_out"][lo:hi])
+
+
+def test_head_sharded_ranks_match_full_evict(api):
+    """The host logic of sharding by KV head with the CUDA backend: two ranks'
+    KV heads of every layer scored separately, their per-head TV masses
+    concatenated in head order (what the all-gather returns), S_l summed in head
+    order -- bit-identical to one full tgvkv_evict's statistic -- budgets from
+    it, each rank's heads selected and gathered on their own, every set equal
+    to the full call's.  The ranks run one after another on one GPU."""
+    from paper_2606_03075_gb300 import shard
+    wl = synth.custom("shard_heads_gpu", 4, 12, 4, 128,
+                      [("text", 11), ("vision", 300), ("text", 9), ("vision", 140),
+                       ("text", 33)], weights="dirichlet", ratios=(0.15,))
+    inp = synth.generate(wl, seed=4)
+    dev = P.device_inputs(inp)
+    full = P.run_evict(api, wl, inp, 0.15, dev)
+    assert full["status"] == 0
+    desc_full = api.desc_for_workload(wl)
+    backend = shard.CudaBackend("cuda")
+    world, G, H = 2, wl.H_q // wl.H_kv, wl.H_kv
+    masses, parts = [], []
+    for r in range(world):
+        g0, g1 = shard.head_range(H, r, world)
+        d = api.make_desc(wl.L, G * (g1 - g0), g1 - g0, wl.d, wl.N, wl.N_v, wl.n_win, 0.0, wl.n_win)
+        s, m = backend.score_heads(d, dev["q"][:, G * g0:G * g1].contiguous(),
+                                   dev["k"][:, g0:g1].contiguous(), dev["modality"],
+                                   dev["text_pos"], dev["w"])
+        masses.append(m)
+        parts.append((g0, g1, d, s))
+    stat = shard.layer_stat_from_heads(torch.cat(masses, dim=1))
+    np.testing.assert_array_equal(stat.cpu().numpy(), full["stat"])
+    budgets = backend.budget(desc_full, stat, 0.15)
+    np.testing.assert_array_equal(budgets.cpu().numpy(), full["budgets"])
+    for g0, g1, d, s in parts:
+        np.testing.assert_array_equal(s.cpu().numpy(), full["scores"][:, g0:g1])
+        off, idx, ko, vo = backend.select_compact(d, s, budgets, dev["modality"],
+                                                  dev["k"][:, g0:g1].contiguous(),
+                                                  dev["v"][:, g0:g1].contiguous())
+        off, idx = off.cpu().numpy(), idx.cpu().numpy()
+        ko, vo = ko.view(torch.int16).cpu().numpy(), vo.view(torch.int16).cpu().numpy()
+        h = g1 - g0
+        for l in range(wl.L):
+            for gl in range(h):
+                lo, hi = off[l * h + gl], off[l * h + gl + 1]
+                rlo, rhi = full["offsets"][l * H + g0 + gl], full["offsets"][l * H + g0 + gl + 1]
+                np.testing.assert_array_equal(idx[lo:hi], full["idx"][rlo:rhi])
+                np.testing.assert_array_equal(ko[lo:hi], full["k_out"][rlo:rhi])
+                np.testing.assert_array_equal(vo[lo:hi], full["v_out"][rlo:rhi])

@@ -145,3 +145,65 @@ def test_a_rank_that_leaves_fails_the_exchange_instead_of_hanging():
         outcome = open(os.path.join(outdir, "r0.txt")).read().split()
         assert outcome[0] == "error", outcome
         assert float(outcome[1]) < 30.0
+
+
+class OracleHeadBackend(OracleBackend):
+    """The oracle with per-head TV masses (for sharding by KV head)."""
+
+    def score_heads(self, desc, q, k, modality, text_pos, w):
+        qd, kd = oracle.widen_bf16(q.numpy()), oracle.widen_bf16(k.numpy())
+        scale = 1.0 / math.sqrt(desc.d)
+        s, _ = oracle.twr_scores_tvb_stat(qd, kd, modality.numpy(), text_pos.numpy(),
+                                          w.numpy().astype(np.float64), scale, desc.H_kv)
+        m = oracle.tv_statistic_per_head(qd, kd, modality.numpy(), text_pos.numpy(), scale,
+                                         desc.H_kv)
+        return torch.from_numpy(s), torch.from_numpy(np.asarray(m, np.float64))
+
+
+WLH = synth.custom("shard_heads", 3, 8, 4, 64, [("text", 9), ("vision", 70), ("text", 6),
+                                                ("vision", 30), ("text", 12)],
+                   weights="dirichlet", ratios=(0.2,))
+
+
+def _rank_heads(rank, world, port, outdir):
+    dist.init_process_group("gloo", init_method=f"tcp://127.0.0.1:{port}", rank=rank,
+                            world_size=world)
+    try:
+        inp = synth.generate(WLH, seed=9)
+        G = WLH.H_q // WLH.H_kv
+        g0, g1 = shard.head_range(WLH.H_kv, rank, world)
+        local = {"q": torch.from_numpy(np.ascontiguousarray(inp["q"][:, G * g0:G * g1])),
+                 "k": torch.from_numpy(np.ascontiguousarray(inp["k"][:, g0:g1])),
+                 "v": torch.from_numpy(np.ascontiguousarray(inp["v"][:, g0:g1])),
+                 "w": torch.from_numpy(inp["w"]),
+                 "modality": torch.from_numpy(inp["modality"]),
+                 "text_pos": torch.from_numpy(inp["text_pos"].astype(np.int32))}
+        res = shard.head_sharded_evict(_desc(WLH), local, 0.2, rank, world, OracleHeadBackend())
+        np.savez(os.path.join(outdir, f"h{rank}.npz"), g0=g0, g1=g1, budgets=res.budgets.numpy(),
+                 stat=res.tvb_stat.numpy(), offsets=res.offsets.numpy(), idx=res.idx.numpy(),
+                 k_out=res.k_out.numpy())
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_cpu_ranks_sharded_by_kv_head_match_the_unsharded_oracle():
+    world = 2
+    inp = synth.generate(WLH, seed=9)
+    ref = oracle.evict(inp["q"], inp["k"], inp["v"], inp["modality"], inp["text_pos"], inp["w"],
+                       0.2, WLH.H_kv)
+    with tempfile.TemporaryDirectory() as outdir:
+        mp.spawn(_rank_heads, args=(world, _free_port(), outdir), nprocs=world, join=True)
+        H = WLH.H_kv
+        for r in range(world):
+            z = np.load(os.path.join(outdir, f"h{r}.npz"))
+            np.testing.assert_array_equal(z["budgets"], ref["budgets"])
+            assert np.allclose(z["stat"], ref["stat"], rtol=1e-12)
+            g0, g1 = int(z["g0"]), int(z["g1"])
+            h = g1 - g0
+            for l in range(WLH.L):
+                for gl in range(h):
+                    g = g0 + gl
+                    lo, hi = z["offsets"][l * h + gl], z["offsets"][l * h + gl + 1]
+                    rlo, rhi = ref["offsets"][l * H + g], ref["offsets"][l * H + g + 1]
+                    np.testing.assert_array_equal(z["idx"][lo:hi], ref["idx"][rlo:rhi])
+                    np.testing.assert_array_equal(z["k_out"][lo:hi], ref["k_out"][rlo:rhi])
