@@ -5,21 +5,34 @@ Prints ONE JSON line on stdout (rank 0).  Metric: eviction microseconds per
 decoder layer for the fused tgvkv_evict over all layers of one request, plus
 the achieved HBM bandwidth of the step and the roofline of its dominant kernel.
 
-  python bench.py [--gpus N --steps K --warmup W] [--config llava15 --ratio 0.05]
+  python bench.py [--gpus N --steps K --warmup W] [--config next --ratio 0.05]
   python bench.py --impl reference ...   (the fp64 CPU oracle, same metric)
+
+The headline line is the LLaVA-NeXT-shaped workload (32 layers, 32/32 heads,
+N = 3008, 788 MB of K: the largest by bytes, where the HBM roof binds) at 5%
+vision retention; the same line carries a `per_config` block with every
+workload and budget (bounded steps each).
 
 Multi-GPU (torchrun, one rank per GPU): every rank runs its own replica of the
 workload (the step has no data-path exchange); the timed region is bracketed by
 a barrier and synchronisation and the max over ranks is reported.
 """
+import os
+import sys
+
+if "reference" in sys.argv[1:]:
+    # the reference arm is the single-threaded oracle: BLAS gets one thread
+    # before numpy is first imported
+    for _k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS",
+               "BLIS_NUM_THREADS", "VECLIB_MAXIMUM_THREADS"):
+        os.environ[_k] = "1"
+
 import argparse
 import ctypes
 import hashlib
 import json
 import math
-import os
 import statistics
-import sys
 import threading
 import time
 
@@ -45,7 +58,7 @@ def parse():
     ap.add_argument("--steps", type=int, default=1000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="tgvkv", choices=["tgvkv", "reference"])
-    ap.add_argument("--config", default="llava15", choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--config", default="next", choices=sorted(synth.WORKLOADS))
     ap.add_argument("--ratio", type=float, default=None)
     ap.add_argument("--layers", type=int, default=0,
                     help="profiling: cut the workload to this many layers (0 = all)")
@@ -56,6 +69,9 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-next-rows", action="store_true",
                     help="skip timing the Eq. 7 / all-token basis / sink variants of the step")
+    ap.add_argument("--no-per-config", action="store_true",
+                    help="skip the per_config block (every workload and budget)")
+    ap.add_argument("--per-config-steps", type=int, default=100)
     ap.add_argument("--record-traffic", metavar="CSV",
                     help="record the DRAM bytes of one kernel launch from `ncu -i REP --page raw "
                          "--csv` output into profiles/traffic.json (for --stage and --config)")
@@ -202,6 +218,42 @@ def measured_peaks():
         return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))), "measured"
     except (OSError, ValueError):
         return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}, "fallback"
+
+
+def kernel_roof(wl, ratio, stage, launch_ms, peaks, peak_src="measured"):
+    """Binding roof of one kernel launch: HBM unless the kernel's algorithmic
+    FLOPs take longer than its bytes at the measured peaks (grouped-query
+    shapes of the score kernel)."""
+    hbm_peak = float(peaks["hbm_gbs"])
+    tensor_peak = float(peaks["bf16_tflops"])
+    nbytes = stage_bytes(wl, ratio)[stage]
+    flops = score_flops(wl) if stage == "score" else 0
+    if flops / (tensor_peak * 1e12) > nbytes / (hbm_peak * 1e9):
+        roof = {"bound": "tensor", "achieved": flops / (launch_ms * 1e-3) / 1e12,
+                "peak": tensor_peak, "unit": "TFLOP/s",
+                "peak_source": f"{peak_src} bf16_tflops (MEASURED_PEAKS.json, burst)"}
+    else:
+        roof = {"bound": "hbm", "achieved": nbytes / (launch_ms * 1e-3) / 1e9,
+                "peak": hbm_peak, "unit": "GB/s",
+                "peak_source": f"{peak_src} hbm_gbs (MEASURED_PEAKS.json)"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["frac_nominal"] = roof["achieved"] / (NOMINAL_HBM_GBS if roof["bound"] == "hbm"
+                                               else NOMINAL_BF16_TFLOPS)
+    roof["bytes_per_launch"] = nbytes
+    roof["flops_per_launch"] = flops
+    return roof
+
+
+def mufu_of(wl, score_ms, clk_mhz):
+    """The score kernel's exponentials against the MUFU rate at the clock seen."""
+    exps = score_exps(wl)
+    m = {"exps_per_launch": exps,
+         "achieved_G_per_s": exps / (score_ms * 1e-3) / 1e9,
+         "peak_G_per_s": MUFU_EX2_PER_CLK_SM * GB300_SMS * clk_mhz * 1e6 / 1e9,
+         "peak_source": f"{MUFU_EX2_PER_CLK_SM} ex2/clk/SM measured x {GB300_SMS} SMs x "
+                        f"{clk_mhz:.0f} MHz median under load"}
+    m["frac"] = m["achieved_G_per_s"] / m["peak_G_per_s"]
+    return m
 
 
 # --------------------------------------------------------------------------
@@ -402,16 +454,101 @@ def run_reference(args, rank, world):
             "ms_per_step": mean * 1e3, "higher_is_better": False, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": workload_config(wl, ratio),
-            "cpu_baseline": {"kind": "oracle", "cores": os.cpu_count(), "value": value,
+            "cpu_baseline": {"kind": "oracle", "cores": 1, "value": value,
                              "unit": UNIT,
                              "sample": f"each step = one (layer, KV head) unit of {wl.name} "
                                        f"(scores of its {wl.G} query heads, TVB split, TPR "
-                                       f"select, gather), fp64 numpy; µs/layer = step "
+                                       f"select, gather), fp64 numpy on one thread (BLAS "
+                                       f"limited to one thread); µs/layer = step "
                                        f"time x H_kv={wl.H_kv}"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
     return 0
+
+
+# --------------------------------------------------------------------------
+# every workload and budget, bounded steps each
+# --------------------------------------------------------------------------
+PER_CONFIG = [("tiny", 0.25), ("llava15", 0.05), ("llava15", 0.20), ("next", 0.05),
+              ("next", 0.10), ("next", 0.20), ("qwen25", 0.05), ("video", 0.05)]
+
+
+def run_per_config(api, torch, dev, stream, barrier, seed, n_steps, inputs=None):
+    """The fused step (tgvkv_evict) and its score kernel alone (tgvkv_score) on
+    every workload and budget: n_steps timed calls each after 3 warm-up calls,
+    inputs rotated past L2.  Returns {"<name> r=<ratio>": {...}} and the clocks
+    seen over the whole block."""
+    peaks, peak_src = measured_peaks()
+    hbm_peak = float(peaks["hbm_gbs"])
+    res = {}
+    with ClockSampler(dev) as clocks:
+        for name in dict.fromkeys(n for n, _ in PER_CONFIG):
+            wl = synth.WORKLOADS[name]
+            inp = (inputs or {}).get(name) or synth.generate(wl, seed=seed)
+            in_bytes = sum(wl.input_bytes().values())
+            n_sets = max(2, math.ceil(2 * L2_BYTES / in_bytes) + 1)
+
+            def up(a, dtype=None):
+                t = torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+                return t.view(dtype) if dtype is not None else t
+
+            sets = [dict(q=up(inp["q"], torch.bfloat16), k=up(inp["k"], torch.bfloat16),
+                         v=up(inp["v"], torch.bfloat16), modality=up(inp["modality"]),
+                         text_pos=up(inp["text_pos"]), w=up(inp["w"])) for _ in range(n_sets)]
+            del inp
+            desc = api.desc_for_workload(wl)
+            ws = api.new_workspace(desc, dev)
+            for cname, ratio in PER_CONFIG:
+                if cname != name:
+                    continue
+                out = api.alloc_outputs(desc, ratio, dev)
+
+                def evict(i):
+                    x = sets[i % n_sets]
+                    api.tgvkv_evict(desc, x["q"], x["k"], x["v"], x["modality"], x["text_pos"],
+                                    x["w"], ratio, out, ws, stream)
+
+                def score(i):
+                    x = sets[i % n_sets]
+                    api.tgvkv_score(desc, x["q"], x["k"], x["modality"], x["text_pos"], x["w"],
+                                    out.scores, out.tvb_stat, ws, stream)
+
+                def timed(call):
+                    for i in range(3):
+                        call(i)
+                    barrier()
+                    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                    a.record(stream)
+                    for i in range(n_steps):
+                        call(3 + i)
+                    b.record(stream)
+                    barrier()
+                    return a.elapsed_time(b) / n_steps      # ms per call
+
+                step_ms = timed(evict)
+                score_ms = timed(score)
+                bits = api.tgvkv_status(ws, stream)
+                if bits != 0:
+                    raise RuntimeError(f"device status bits 0x{bits:x} in {name} r={ratio}")
+                sbytes, rows = step_bytes(wl, ratio)
+                step_gbs = sbytes / (step_ms * 1e-3) / 1e9
+                roof = kernel_roof(wl, ratio, "score", score_ms, peaks, peak_src)
+                clk = clocks.summary().get("sm_mhz") or float(peaks.get("sm_max_mhz", 2070.0))
+                res[f"{name} r={ratio}"] = {
+                    "us_per_layer": step_ms * 1e3 / wl.L, "step_ms": step_ms,
+                    "step_bytes": sbytes, "step_gbs": step_gbs, "step_frac": step_gbs / hbm_peak,
+                    "score_kernel": {"launch_ms": score_ms, "bound": roof["bound"],
+                                     "achieved": roof["achieved"], "unit": roof["unit"],
+                                     "peak": roof["peak"], "frac": roof["frac"],
+                                     "share_of_step": score_ms / step_ms,
+                                     "traffic": recorded_traffic("score", name)},
+                    "score_mufu_frac": mufu_of(wl, score_ms, clk)["frac"],
+                    "tail_ms": step_ms - score_ms, "rows_kept": rows, "steps": n_steps}
+                del out
+            del sets, ws
+            torch.cuda.empty_cache()
+    return res, clocks.summary()
 
 
 # --------------------------------------------------------------------------
@@ -747,37 +884,24 @@ def main():
     # ---- roofline of the dominant kernel and of the whole step
     peaks, peak_src = measured_peaks()
     hbm_peak = float(peaks["hbm_gbs"])
-    tensor_peak = float(peaks["bf16_tflops"])
-    sb = stage_bytes(wl, ratio)
     dom = max(stages, key=lambda s: stage_ms[s])
     traffic = recorded_traffic(dom, wl.name)
-    # the binding roof: HBM unless the kernel's algorithmic FLOPs take longer
-    # than its bytes at the respective measured peaks (grouped-query shapes)
-    flops = score_flops(wl) if dom == "score" else 0
-    if flops / (tensor_peak * 1e12) > sb[dom] / (hbm_peak * 1e9):
-        roof = {"bound": "tensor", "achieved": flops / (stage_ms[dom] * 1e-3) / 1e12,
-                "peak": tensor_peak, "unit": "TFLOP/s",
-                "peak_source": f"{peak_src} bf16_tflops (MEASURED_PEAKS.json, burst)"}
-    else:
-        roof = {"bound": "hbm", "achieved": sb[dom] / (stage_ms[dom] * 1e-3) / 1e9,
-                "peak": hbm_peak, "unit": "GB/s",
-                "peak_source": f"{peak_src} hbm_gbs (MEASURED_PEAKS.json)"}
-    roof["frac"] = roof["achieved"] / roof["peak"]
-    roof["frac_nominal"] = roof["achieved"] / (NOMINAL_HBM_GBS if roof["bound"] == "hbm"
-                                               else NOMINAL_BF16_TFLOPS)
-    # the exponentials of the score kernel against the MUFU rate at the clock seen
+    roof = kernel_roof(wl, ratio, dom, stage_ms[dom], peaks, peak_src)
     clk_mhz = clocks.summary().get("sm_mhz") or float(peaks.get("sm_max_mhz", 2070.0))
-    exps = score_exps(wl)
-    mufu = {"exps_per_launch": exps,
-            "achieved_G_per_s": exps / (stage_ms["score"] * 1e-3) / 1e9,
-            "peak_G_per_s": MUFU_EX2_PER_CLK_SM * GB300_SMS * clk_mhz * 1e6 / 1e9,
-            "peak_source": f"{MUFU_EX2_PER_CLK_SM} ex2/clk/SM measured x {GB300_SMS} SMs x "
-                           f"{clk_mhz:.0f} MHz median under load"}
-    mufu["frac"] = mufu["achieved_G_per_s"] / mufu["peak_G_per_s"]
+    mufu = mufu_of(wl, stage_ms["score"], clk_mhz)
     sbytes, rows = step_bytes(wl, ratio)
     step_gbs = sbytes * args.steps * world / (region_ms * 1e-3) / 1e9
     fbytes = full_step_bytes(wl, ratio)
     full_gbs = fbytes * args.steps * world / (region_ms * 1e-3) / 1e9
+
+    # ---- every workload and budget (the main workload's inputs reused)
+    per_config, per_config_clocks = None, None
+    if not args.no_per_config and not args.layers:
+        del sets
+        torch.cuda.empty_cache()
+        per_config, per_config_clocks = run_per_config(
+            api, torch, dev, stream, barrier, args.seed + rank, args.per_config_steps,
+            inputs={wl.name: inp})
 
     line = None
     if rank == 0:
@@ -804,8 +928,9 @@ def main():
                                             "rows read, idx and offsets"},
             "roofline": {"bound": roof["bound"], "kernel": dom, "achieved": roof["achieved"],
                          "peak": roof["peak"], "unit": roof["unit"], "frac": roof["frac"],
-                         "traffic": traffic, "bytes_per_launch": sb[dom],
-                         "flops_per_launch": flops, "launch_ms": stage_ms[dom],
+                         "traffic": traffic, "bytes_per_launch": roof["bytes_per_launch"],
+                         "flops_per_launch": roof["flops_per_launch"],
+                         "launch_ms": stage_ms[dom],
                          "peak_source": roof["peak_source"], "frac_nominal": roof["frac_nominal"]},
             "score_mufu": mufu,
             "stage_ms": stage_ms,
@@ -819,6 +944,8 @@ def main():
             "e2e": e2e,
             "gpu_launches": launches_per_step * args.steps,
             "clocks": clocks.summary(),
+            "per_config": per_config,
+            "per_config_clocks": per_config_clocks,
         }
     if world > 1:
         dist.barrier()

@@ -93,7 +93,7 @@ extern "C" {
 #define TGVKV_STATUS_TEXT_POS     0x01u /* text_pos not strictly ascending or outside [0, N) */
 #define TGVKV_STATUS_VISION_COUNT 0x02u /* modality marks a vision count other than N_v */
 #define TGVKV_STATUS_BUDGET       0x04u /* a layer budget outside [0, N_v] reached select */
-#define TGVKV_STATUS_INDEX        0x08u /* an index outside [0, N) reached compact */
+#define TGVKV_STATUS_INDEX        0x08u /* compact: an index outside [0, N), or a CSR larger than the output */
 #define TGVKV_STATUS_COUNT        0x10u /* a retained set did not hold N_t + b_l rows */
 #define TGVKV_STATUS_TIMEOUT      0x20u /* a bounded on-chip wait gave up */
 #define TGVKV_STATUS_WEIGHT       0x40u /* a text weight is negative or not finite */
@@ -221,10 +221,16 @@ int tgvkv_select_tpr(const tgvkv_desc* desc, const float* scores, const float* t
 /* Compaction: row r of set (l, g) of the CSR becomes
  *   k_out[r] = k[l][g][idx[r]],  v_out[r] = v[l][g][idx[r]]
  * as bit copies.  k, v: bf16 [L][H_kv][N][d]; k_out, v_out: bf16
- * [offsets[L*H_kv]][d] (output; capacity tgvkv_retained_rows rows). */
+ * [capacity_rows][d] (output; rows 0 .. offsets[L*H_kv] are written, and
+ * tgvkv_retained_rows rows always suffice for sets tgvkv_select made).
+ * capacity_rows: rows the caller allocated in each of k_out and v_out (>= 0).
+ * A CSR whose total offsets[L*H_kv] is negative or above capacity_rows sets
+ * TGVKV_STATUS_INDEX and only rows below capacity_rows are written; an
+ * idx entry outside [0, N) sets the same bit and its row is skipped. */
 int tgvkv_compact(const tgvkv_desc* desc, const uint16_t* k, const uint16_t* v,
                   const int64_t* offsets, const int32_t* idx,
-                  uint16_t* k_out, uint16_t* v_out, void* workspace, void* stream);
+                  uint16_t* k_out, uint16_t* v_out, int64_t capacity_rows,
+                  void* workspace, void* stream);
 
 /* score -> budget -> select -> compact in one stream-ordered call with no host
  * synchronisation.  Arguments as in the four calls above.  With Eq. 7 weights
@@ -347,20 +353,29 @@ const char* tgvkv_last_error(void);
  * - A problem whose scratch exceeds TGVKV_NOALLOC_SCRATCH_BYTES (see
  *   tgvkv_workspace_size) is rejected with TGVKV_ERR_UNSUPPORTED before any
  *   launch.
- * - The first call on each device looks up the array's device address (with
- *   that device current) and caches it; make that first call before any
- *   stream capture.
+ * - Every call looks up the array's device address in the current device's
+ *   context (so a context created after cudaDeviceReset uses its own array);
+ *   the first call on a device may load the library's device code, so make it
+ *   before any stream capture.
  * - All calls share the one array.  Each call clears the parts that must start
  *   at zero; calls whose work overlaps on the GPU (different streams, or
  *   different host threads, on one device) race on the array and must be
  *   serialised by the caller.
- * - The device status word is kept in the array and cleared by every call, so
- *   data-dependent input faults are skipped (never out of bounds) but not
- *   reported; use tgvkv_score with a workspace to read them. */
+ * - The device status word is kept in the array: each call clears it before
+ *   its launch, so after a call tgvkv_noalloc_status returns that call's
+ *   TGVKV_STATUS_* bits (input faults that were skipped, and
+ *   TGVKV_STATUS_TIMEOUT when a bounded wait gave up and the scores are
+ *   unfinished).  Read it before the next call clears it. */
 #define TGVKV_NOALLOC_SCRATCH_BYTES (8u << 20)
 int tgvkv_score_noalloc(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* k,
                         const uint8_t* modality, const int32_t* text_pos, const float* w,
                         float* scores, float* tvb_stat, void* stream);
+
+/* Synchronise `stream`, then read and clear the status word of
+ * tgvkv_score_noalloc's fixed array on the current device (the counterpart of
+ * tgvkv_status for that call).  Returns the TGVKV_STATUS_* bits (0 = clean)
+ * or a negative error code.  Allocates nothing. */
+int tgvkv_noalloc_status(void* stream);
 
 #ifdef __cplusplus
 }

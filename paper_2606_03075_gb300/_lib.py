@@ -46,8 +46,8 @@ SIGNATURES = {
                              c_void_p, c_void_p]),
     "tgvkv_select_tpr": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                  c_void_p, c_void_p, c_void_p]),
-    "tgvkv_compact": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
-                              c_void_p, c_void_p, c_void_p]),
+    "tgvkv_compact": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                              c_int64, c_void_p, c_void_p]),
     "tgvkv_evict": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                             c_double, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                             c_void_p, c_void_p, c_void_p, c_void_p]),
@@ -67,6 +67,7 @@ SIGNATURES = {
     "tgvkv_last_error": (c_char_p, []),
     "tgvkv_score_noalloc": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                     c_void_p, c_void_p, c_void_p]),
+    "tgvkv_noalloc_status": (c_int, [c_void_p]),
 }
 
 _lib = None

@@ -200,12 +200,14 @@ def tgvkv_select_tpr(desc, scores, text_scores, budgets, modality, offsets, idx,
 
 def tgvkv_compact(desc, k, v, offsets, idx, k_out, v_out, ws, stream=None):
     n = desc.L * desc.H_kv * desc.N * desc.d
+    capacity = min(k_out.numel(), v_out.numel()) // desc.d   # rows of the outputs
     _check(_lib.load().tgvkv_compact(
         ctypes.byref(desc),
         _ptr(k, _BF16_LIKE, n, "k"), _ptr(v, _BF16_LIKE, n, "v"),
         _ptr(offsets, (torch.int64,), desc.L * desc.H_kv + 1, "offsets"),
         _ptr(idx, (torch.int32,), 0, "idx"),
         _ptr(k_out, _BF16_LIKE, 0, "k_out"), _ptr(v_out, _BF16_LIKE, 0, "v_out"),
+        capacity,
         _ptr(ws, (torch.uint8,), tgvkv_workspace_size(desc), "workspace"),
         _stream(stream)), "tgvkv_compact")
 

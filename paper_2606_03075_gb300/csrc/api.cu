@@ -5,7 +5,7 @@
 #include <stdio.h>
 #include <string.h>
 
-#include <mutex>
+#include <algorithm>
 
 #include "common.cuh"
 #include "launch.h"
@@ -429,10 +429,12 @@ int tgvkv_select(const tgvkv_desc* desc, const float* scores, const int32_t* bud
 
 int tgvkv_compact(const tgvkv_desc* desc, const uint16_t* k, const uint16_t* v,
                   const int64_t* offsets, const int32_t* idx, uint16_t* k_out, uint16_t* v_out,
-                  void* workspace, void* stream) {
+                  int64_t capacity_rows, void* workspace, void* stream) {
     Problem p{};
     int rc = make_problem(desc, &p);
     if (rc) return rc;
+    if (capacity_rows < 0) return fail(TGVKV_ERR_INVALID_ARG, "capacity_rows %lld < 0",
+                                       (long long)capacity_rows);
     REQUIRE_PTR(k, "k", true);
     REQUIRE_PTR(v, "v", true);
     REQUIRE_PTR(offsets, "offsets", false);
@@ -441,8 +443,8 @@ int tgvkv_compact(const tgvkv_desc* desc, const uint16_t* k, const uint16_t* v,
     REQUIRE_PTR(v_out, "v_out", true);
     REQUIRE_PTR(workspace, "workspace", true);
     const WsLayout lay = layout_of(p);
-    // every set holds at most N rows
-    const long long cap = (long long)p.L * p.H_kv * p.N;
+    // every set holds at most N rows: no more can be asked of the kernel
+    const long long cap = std::min((long long)capacity_rows, (long long)p.L * p.H_kv * p.N);
     cudaError_t e = launch_compact(p, k, v, offsets, idx, k_out, v_out, cap,
                                    status_of(workspace, lay), static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? ok() : cuda_fail(e, "compact launch");
@@ -574,28 +576,16 @@ namespace {
 // previous call's contents; the call clears what must start at zero.
 static __device__ __align__(256) unsigned char g_noalloc_scratch[TGVKV_NOALLOC_SCRATCH_BYTES];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_noalloc_mutex;
-void* g_noalloc_ptr[kMaxDevices] = {};
-
-// Device address of g_noalloc_scratch on the current device, looked up once per
-// device.  The name is a host-side stand-in: only this address may be given to
-// a kernel.
+// Device address of g_noalloc_scratch in the current device's context.  The
+// name is a host-side stand-in: only this address may be given to a kernel.
+// It is looked up on every call (a cheap query once the module is loaded), so
+// a context created after cudaDeviceReset gets its own array's address.
 int noalloc_scratch(void** out) {
-    int dev = -1;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return tgvkv::cuda_fail(e, "cudaGetDevice");
-    if (dev < 0 || dev >= kMaxDevices)
-        return tgvkv::fail(TGVKV_ERR_UNSUPPORTED, "device ordinal %d above %d", dev, kMaxDevices);
-    std::lock_guard<std::mutex> lock(g_noalloc_mutex);
-    if (!g_noalloc_ptr[dev]) {
-        void* ptr = nullptr;
-        e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
-        if (e != cudaSuccess || ptr == nullptr)
-            return tgvkv::cuda_fail(e, "cudaGetSymbolAddress(static scratch)");
-        g_noalloc_ptr[dev] = ptr;
-    }
-    *out = g_noalloc_ptr[dev];
+    void* ptr = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
+    if (e != cudaSuccess || ptr == nullptr)
+        return tgvkv::cuda_fail(e, "cudaGetSymbolAddress(static scratch)");
+    *out = ptr;
     return TGVKV_OK;
 }
 
@@ -627,4 +617,12 @@ extern "C" int tgvkv_score_noalloc(const tgvkv_desc* desc, const uint16_t* q_tex
     if (e != cudaSuccess) return cuda_fail(e, "static scratch clear");
     rc = do_score(p, q_text, k, modality, text_pos, w, scores, tvb_stat, scratch, st);
     return rc ? rc : ok();
+}
+
+extern "C" int tgvkv_noalloc_status(void* stream) {
+    void* scratch = nullptr;
+    int rc = noalloc_scratch(&scratch);
+    if (rc) return -rc;
+    // the status word sits at offset 0 of every workspace layout
+    return tgvkv_status(scratch, stream);
 }

@@ -16,12 +16,18 @@ template <int VPR>  // 16-byte vectors per row: d * 2 / 16
 __global__ void __launch_bounds__(kThreads)
 compact_kernel(Problem p, const uint4* __restrict__ k, const uint4* __restrict__ v,
                const int64_t* __restrict__ offsets, const int32_t* __restrict__ idx,
-               uint4* __restrict__ k_out, uint4* __restrict__ v_out, uint32_t* __restrict__ status) {
+               uint4* __restrict__ k_out, uint4* __restrict__ v_out, long long capacity,
+               uint32_t* __restrict__ status) {
     constexpr int RPI = 32 / VPR;                 // rows per warp per iteration
     constexpr int ROWS_PER_WARP = RPI * kIter;
     constexpr int ROWS_PER_CTA = ROWS_PER_WARP * (kThreads / 32);
     const int n_heads = p.L * p.H_kv;
-    const long long total = offsets[n_heads];
+    long long total = offsets[n_heads];
+    if (total < 0 || total > capacity) {
+        // a CSR that does not fit the output: write the rows that do
+        if (blockIdx.x == 0 && threadIdx.x == 0) raise_status(status, TGVKV_STATUS_INDEX);
+        total = total < 0 ? 0 : capacity;
+    }
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const long long r0 = (long long)blockIdx.x * ROWS_PER_CTA + (long long)warp * ROWS_PER_WARP;
     if (r0 >= total) return;
@@ -75,7 +81,7 @@ cudaError_t launch_compact_t(const Problem& p, const uint16_t* k, const uint16_t
     if (blocks == 0) return cudaSuccess;
     compact_kernel<VPR><<<(unsigned)blocks, kThreads, 0, stream>>>(
         p, reinterpret_cast<const uint4*>(k), reinterpret_cast<const uint4*>(v), offsets, idx,
-        reinterpret_cast<uint4*>(k_out), reinterpret_cast<uint4*>(v_out), status);
+        reinterpret_cast<uint4*>(k_out), reinterpret_cast<uint4*>(v_out), capacity_rows, status);
     return cudaGetLastError();
 }
 

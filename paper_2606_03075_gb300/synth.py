@@ -29,6 +29,8 @@ channels).  Queries and values are iid N(0, 1).  Everything is rounded to bf16
 """
 from __future__ import annotations
 
+import os
+from concurrent.futures import ThreadPoolExecutor
 from dataclasses import dataclass, field
 
 import numpy as np
@@ -169,6 +171,18 @@ def draw_layer(wl: Workload, seed: int, layer: int):
     return to_bf16_bits(q), to_bf16_bits(k), to_bf16_bits(v), w
 
 
+def _each_layer(fn, n_layers):
+    """fn(l) for every layer on a few threads (every layer draws from its own
+    seeded streams, so the result does not depend on the order)."""
+    workers = max(1, min(n_layers, os.cpu_count() or 1, 16))
+    if workers == 1:
+        for l in range(n_layers):
+            fn(l)
+        return
+    with ThreadPoolExecutor(workers) as ex:
+        list(ex.map(fn, range(n_layers)))
+
+
 def generate(wl: Workload, seed: int = 0) -> dict:
     """All inputs of one eviction step as host numpy arrays."""
     L, n, d, n_win = wl.L, wl.N, wl.d, wl.n_win
@@ -176,8 +190,11 @@ def generate(wl: Workload, seed: int = 0) -> dict:
     k = np.empty((L, wl.H_kv, n, d), np.int16)
     v = np.empty((L, wl.H_kv, n, d), np.int16)
     w = np.empty((L, n_win), np.float32)
-    for l in range(L):
+
+    def one(l):
         q[l], k[l], v[l], w[l] = draw_layer(wl, seed, l)
+
+    _each_layer(one, L)
     return dict(q=q, k=k, v=v, w=w, modality=wl.modality,
                 text_pos=wl.text_pos.astype(np.int32))
 
@@ -197,8 +214,11 @@ def generate_prefill(wl: Workload, seed: int = 0, inp: dict | None = None) -> di
     rows at the query positions are generate()'s q."""
     inp = dict(inp if inp is not None else generate(wl, seed))
     q_all = np.empty((wl.L, wl.H_q, wl.N, wl.d), np.int16)
-    for l in range(wl.L):
+
+    def one(l):
         q_all[l] = draw_prefill_queries(wl, seed, l, inp["q"][l])
+
+    _each_layer(one, wl.L)
     inp["q_all"] = q_all
     return inp
 

@@ -117,3 +117,66 @@ def gap_rule(ref, b, idx, off, modality, gpu_scores):
             f"{kth - nxt!r} (k-th {kth!r})")
         for v in kept ^ want:
             assert abs(ref[g][v] - kth) <= RTOL * abs(kth) + 1e-12, (g, v, ref[g][v], kth)
+
+
+# ---------------------------------------------------------------- every layer
+_STAT_CACHE = {}
+
+
+def oracle_stat_all_layers(wl, inp, seed_key=None):
+    """fp64 oracle statistic S_l of every layer, [L]; one spawned process per
+    core (never forked: the test process has used the GPU).  Cached per
+    workload and seed key."""
+    key = (wl.name, seed_key)
+    if key in _STAT_CACHE:
+        return _STAT_CACHE[key]
+    import concurrent.futures as cf
+    import multiprocessing as mp
+    import os
+    scale = 1.0 / math.sqrt(wl.d)
+    jobs = [(inp["q"][l], inp["k"][l], inp["modality"], inp["text_pos"], inp["w"][l], scale,
+             wl.H_kv) for l in range(wl.L)]
+    workers = max(1, min(wl.L, os.cpu_count() or 1))
+    import _oracle_workers
+    one = ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS")
+    saved = {k: os.environ.get(k) for k in one}
+    os.environ.update({k: "1" for k in one})     # one BLAS thread per worker process
+    try:
+        with cf.ProcessPoolExecutor(workers, mp_context=mp.get_context("spawn")) as ex:
+            stat = np.array(list(ex.map(_oracle_workers.layer_stat, jobs)))
+    finally:
+        for k, v in saved.items():
+            if v is None:
+                os.environ.pop(k, None)
+            else:
+                os.environ[k] = v
+    _STAT_CACHE[key] = stat
+    return stat
+
+
+def budgets_match(gpu_budgets, ref_stat, total, cap, rtol=RTOL):
+    """The GPU's budgets against oracle.tvb_budgets on the oracle's fp64
+    statistic.  They must be equal, except for layers whose quota (Eq. 5) sits
+    within the tolerance of a rounding boundary: a statistic within rtol of the
+    oracle's moves each quota by at most about 2 rtol of itself, so a layer may
+    differ (by one unit) only where its fractional part is that close to an
+    integer or to another layer's fractional part (the largest-remainder cut).
+    Returns the layers that differ."""
+    gpu = np.asarray(gpu_budgets, np.int64)
+    want = np.asarray(oracle.tvb_budgets(ref_stat, total, cap), np.int64)
+    assert gpu.sum() == want.sum() == total
+    diff = np.flatnonzero(gpu != want)
+    if diff.size == 0:
+        return []
+    stat = np.asarray(ref_stat, np.float64)
+    quota = total * stat / stat.sum()
+    frac = quota - np.floor(quota)
+    tol = 2 * rtol * quota
+    for l in diff:
+        assert abs(int(gpu[l]) - int(want[l])) == 1, (l, gpu[l], want[l])
+        near_int = min(frac[l], 1.0 - frac[l]) <= tol[l]
+        near_other = np.any(np.abs(np.delete(frac, l) - frac[l]) <= np.delete(tol, l) + tol[l])
+        assert near_int or near_other, (
+            f"layer {l}: budget {gpu[l]} != oracle {want[l]} though its quota {quota[l]!r} "
+            f"is not within tolerance of a rounding boundary")
+    return diff.tolist()

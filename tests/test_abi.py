@@ -67,7 +67,8 @@ def test_validation_rejects_before_launch(lib):
     assert lib.tgvkv_budget(ref(d), fake, -0.1, fake, fake, None) == 1
     assert lib.tgvkv_budget(ref(d), fake, float("nan"), fake, fake, None) == 1
     assert lib.tgvkv_select(ref(d), fake, fake, fake, fake, P(0), fake, None) == 1
-    assert lib.tgvkv_compact(ref(d), fake, fake, fake, fake, odd, fake, fake, None) == 1
+    assert lib.tgvkv_compact(ref(d), fake, fake, fake, fake, odd, fake, 10, fake, None) == 1
+    assert lib.tgvkv_compact(ref(d), fake, fake, fake, fake, fake, fake, -1, fake, None) == 1
     assert lib.tgvkv_evict(ref(d), fake, fake, fake, fake, fake, fake, 2.0, fake, fake, fake,
                            fake, fake, fake, fake, fake, None) == 1
     assert lib.tgvkv_workspace_size(ref(_desc(d=32))) == 0
