@@ -92,6 +92,22 @@ def workload_of(args):
     return wl
 
 
+def rotation_sets(wl):
+    """Input sets the GPU arm rotates through so that every step's inputs
+    miss L2 (their total is above twice the L2 size)."""
+    in_bytes = sum(wl.input_bytes().values())
+    return max(2, math.ceil(2 * L2_BYTES / in_bytes) + 1), in_bytes
+
+
+def full_config(wl, ratio, world):
+    """The `config` of a bench line (both arms)."""
+    n_sets, in_bytes = rotation_sets(wl)
+    return dict(workload_config(wl, ratio),
+                l2="inputs larger than L2: %d rotating input sets of %.0f MB "
+                   "(L2 %d MB)" % (n_sets, in_bytes / 1e6, L2_BYTES >> 20),
+                parallelism=f"replicas x{world}")
+
+
 def workload_config(wl, ratio):
     return {"workload": f"{wl.name}: L={wl.L} H_q/H_kv={wl.H_q}/{wl.H_kv} d={wl.d} "
                         f"N={wl.N} (N_v={wl.N_v}, N_t={wl.N_t}) query rows={wl.n_win} "
@@ -453,7 +469,7 @@ def run_reference(args, rank, world):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": mean * 1e3, "higher_is_better": False, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": workload_config(wl, ratio),
+            "config": full_config(wl, ratio, world),
             "cpu_baseline": {"kind": "oracle", "cores": 1, "value": value,
                              "unit": UNIT,
                              "sample": f"each step = one (layer, KV head) unit of {wl.name} "
@@ -580,8 +596,7 @@ def main():
     ratio = args.ratio if args.ratio is not None else wl.ratios[0]
     desc = api.desc_for_workload(wl)
     inp = synth.generate(wl, seed=args.seed + rank)
-    in_bytes = sum(wl.input_bytes().values())
-    n_sets = max(2, math.ceil(2 * L2_BYTES / in_bytes) + 1)
+    n_sets, in_bytes = rotation_sets(wl)
 
     def upload(a, dtype=None):
         t = torch.from_numpy(np.ascontiguousarray(a)).to(dev)
@@ -914,10 +929,7 @@ def main():
             "ms_per_step": region_ms / args.steps, "higher_is_better": False,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16->f32",
             "data": "synthetic",
-            "config": dict(workload_config(wl, ratio),
-                           l2="inputs larger than L2: %d rotating input sets of %.0f MB "
-                              "(L2 %d MB)" % (n_sets, in_bytes / 1e6, L2_BYTES >> 20),
-                           parallelism=f"replicas x{world}"),
+            "config": full_config(wl, ratio, world),
             "hbm_step": {"bytes_per_step": sbytes, "bytes_per_layer": sbytes / wl.L,
                          "gbs": step_gbs, "peak": hbm_peak, "frac": step_gbs / hbm_peak,
                          "frac_nominal": step_gbs / NOMINAL_HBM_GBS,
