@@ -176,7 +176,7 @@ def score_flops(wl):
 
 # each kernel's source with the headers it includes (a change to any of them
 # invalidates a recorded ncu traffic figure)
-KERNEL_SOURCES = {"score": ("score_tc.cu", "score_cl.cu", "rowstat.cuh", "tc05.cuh", "common.cuh"),
+KERNEL_SOURCES = {"score": ("score_tc.cu", "rowstat.cuh", "tc05.cuh", "common.cuh"),
                   "budget": ("budget.cu", "budget.cuh", "common.cuh"),
                   "select": ("select.cu", "budget.cuh", "common.cuh"),
                   "compact": ("compact.cu", "common.cuh")}

@@ -20,7 +20,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libtgvkv.so")
 
-SOURCES = ["api.cu", "score_tc.cu", "score_cl.cu", "budget.cu", "select.cu", "compact.cu", "text.cu", "decode.cu",
+SOURCES = ["api.cu", "score_tc.cu", "budget.cu", "select.cu", "compact.cu", "text.cu", "decode.cu",
            "prefill.cu", "selftest.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",

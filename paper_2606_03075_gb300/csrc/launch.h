@@ -20,15 +20,6 @@ cudaError_t launch_score(const Problem& p, const uint16_t* q, const uint16_t* k,
                          float* scores, float* tvb_stat, char* ws, const WsLayout& lay,
                          long long budget_total, int32_t* budgets, cudaStream_t stream);
 
-// The score kernel for heads of one row tile whose keys are split over a
-// thread-block cluster and kept resident in shared memory (score_cl.cu);
-// launch_score dispatches to it when score_cluster_eligible(p).
-bool score_cluster_eligible(const Problem& p);
-cudaError_t launch_score_cluster(const Problem& p, const uint16_t* q, const uint16_t* k,
-                                 const uint8_t* modality, const int32_t* text_pos, const float* w,
-                                 float* scores, float* tvb_stat, char* ws, const WsLayout& lay,
-                                 long long budget_total, int32_t* budgets, cudaStream_t stream);
-
 // TVB split of `total` (budget.cu); the cap is N_v (vision basis) or N.
 cudaError_t launch_budget(const Problem& p, const float* tvb_stat, long long total,
                           int32_t* budgets, uint32_t* status, cudaStream_t stream);

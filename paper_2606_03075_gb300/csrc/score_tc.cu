@@ -1064,9 +1064,6 @@ cudaError_t launch_score(const Problem& p, const uint16_t* q, const uint16_t* k,
         if (e == cudaSuccess) e = cudaMemsetAsync(tvb_stat, 0, sizeof(float) * units, stream);
         return e;
     }
-    if (score_cluster_eligible(p))
-        return launch_score_cluster(p, q, k, modality, text_pos, w, scores, tvb_stat, ws, lay,
-                                    budget_total, budgets, stream);
     if (p.d == 64)
         return launch_tc<64>(p, q, k, modality, text_pos, w, scores, tvb_stat, ws, lay, budget_total,
                              budgets, stream);

@@ -52,35 +52,34 @@ SMALL = {
 }
 
 
-# Heads of one row tile with 64 < G * n_win <= 128 and d = 128: the score kernel
-# that splits each head's keys over a thread-block cluster (1 to 8 CTAs here,
-# 6 at the next workload's full size) and keeps them in shared memory.
-CLUSTER = {
-    # one CTA holds a whole head; grouped-query heads (G = 2, 96 rows)
-    "cl1_gqa": synth.custom("cl1_gqa", 2, 8, 4, 128,
+# Heads of one row tile with 64 < G * n_win <= 128 and d = 128 (the score
+# kernel's single-tile items) at several lengths, row counts and causal layouts.
+ONE_TILE = {
+    # grouped-query heads (G = 2, 96 rows)
+    "gqa_96": synth.custom("gqa_96", 2, 8, 4, 128,
                             [("text", 11), ("vision", 400), ("text", 6), ("vision", 50),
                              ("text", 48)], ratios=(0.1,)),
-    # two CTAs, 80 rows; vision keys after the last query row (scores 0)
-    "cl2_r80_tail": synth.custom("cl2_r80_tail", 3, 4, 4, 128,
+    # 80 rows; vision keys after the last query row (scores 0)
+    "r80_tail": synth.custom("r80_tail", 3, 4, 4, 128,
                                  [("text", 10), ("vision", 700), ("text", 80), ("vision", 300)],
                                  window=80, ratios=(0.2,)),
-    # three CTAs, 112 rows (G = 7), Dirichlet weights, ragged N
-    "cl3_r112": synth.custom("cl3_r112", 2, 14, 2, 128,
+    # 112 rows (G = 7), Dirichlet weights, ragged N
+    "r112_dirichlet": synth.custom("r112_dirichlet", 2, 14, 2, 128,
                              [("text", 7), ("vision", 900), ("text", 5), ("vision", 611),
                               ("text", 16)], window=16, weights="dirichlet", ratios=(0.05,)),
-    # four CTAs, 128 rows spread over the sequence (rows see different key prefixes)
-    "cl4_r128_causal": synth.custom("cl4_r128_causal", 2, 2, 2, 128,
+    # 128 rows spread over the sequence (rows see different key prefixes)
+    "r128_causal": synth.custom("r128_causal", 2, 2, 2, 128,
                                     [("text", 20), ("vision", 500), ("text", 40), ("vision", 500),
                                      ("text", 40), ("vision", 500), ("text", 48)], window=128,
                                     ratios=(0.1,)),
-    # many items per cluster (256 heads), two CTAs
-    "cl_many": synth.custom("cl_many", 8, 32, 32, 128,
+    # many heads (256) per launch
+    "many_heads_96": synth.custom("many_heads_96", 8, 32, 32, 128,
                             [("text", 30), ("vision", 700), ("text", 96)], ratios=(0.1,)),
-    # a cluster of one CTA (short heads)
-    "cl_one_cta": synth.custom("cl_one_cta", 2, 4, 4, 128,
+    # short heads
+    "short_96": synth.custom("short_96", 2, 4, 4, 128,
                                [("text", 10), ("vision", 154), ("text", 96)], ratios=(0.25,)),
-    # eight CTAs, 128 rows (three pass-B buffers), ragged N
-    "cl8_r128": synth.custom("cl8_r128", 1, 4, 2, 128,
+    # 128 rows, long heads, ragged N
+    "long_r128": synth.custom("long_r128", 1, 4, 2, 128,
                              [("text", 17), ("vision", 2800), ("text", 64)], window=64,
                              ratios=(0.05,)),
 }
@@ -120,12 +119,12 @@ def test_small_layouts(api, name):
         _full_check(api, wl, r)
 
 
-@pytest.mark.parametrize("name", sorted(CLUSTER))
-def test_cluster_layouts(api, name):
+@pytest.mark.parametrize("name", sorted(ONE_TILE))
+def test_one_tile_layouts(api, name):
     """The whole step against the oracle, then the score call alone (scores
     and statistic within tolerance, no budgets) and a second evict call
     bit-identical to the first."""
-    wl = CLUSTER[name]
+    wl = ONE_TILE[name]
     inp = synth.generate(wl, seed=3)
     g, ref = _full_check(api, wl, wl.ratios[0], inp=inp)
     dev = P.device_inputs(inp)
