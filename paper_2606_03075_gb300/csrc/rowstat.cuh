@@ -118,10 +118,59 @@ __device__ __forceinline__ void exp_word_both(const float (&x)[32], float sl2, f
 }
 
 // Online statistics of one row over one 32-key word: columns 0..lim visible.
-// row_word with the complement mass u as well (text-key pass).
+// The row keeps a reference m (base-2 units) and sums its terms 2^(x sl2 - m):
+// the row's first visible word sets m to that word's maximum; a later word
+// keeps m unless its terms against m sum above kWordSumLimit (some term large,
+// or overflowed), and is then taken again against its own maximum, which moves
+// m up (z and v rescaled).  Any reference gives the same attention entries
+// 2^(x sl2 - m) / Z; this one never exceeds the row's maximum and keeps every
+// term at most kWordSumLimit, and most words skip the 32-key maximum.
+constexpr float kWordSumLimit = 32.f * 256.f;
+
+__device__ __forceinline__ void row_word(const float (&x)[32], float sl2, int lim, uint32_t vm,
+                                         float& m, float& z, float& v) {
+    if (lim < 0) return;
+    if (m != -INFINITY) {
+        float zs = 0.f, vs = 0.f;
+        if (lim >= 31)
+            exp_word<false>(x, sl2, -m, 31, vm, zs, vs);
+        else
+            exp_word<true>(x, sl2, -m, lim, vm, zs, vs);
+        if (zs <= kWordSumLimit) {   // false for inf and nan too
+            z += zs;
+            v += vs;
+            return;
+        }
+    }
+    const float m_new = fmaxf(m, (lim >= 31 ? max32(x) : max32_masked(x, lim)) * sl2);
+    const float alpha = fast_exp2(m - m_new);   // m = -inf: alpha = 0, z = v = 0 stay 0
+    z *= alpha;
+    v *= alpha;
+    if (lim >= 31)
+        exp_word<false>(x, sl2, -m_new, 31, vm, z, v);
+    else
+        exp_word<true>(x, sl2, -m_new, lim, vm, z, v);
+    m = m_new;
+}
+
+// row_word with the complement mass u as well (text-key pass: the visible keys
+// not in vm).
 __device__ __forceinline__ void row_word_both(const float (&x)[32], float sl2, int lim, uint32_t vm,
                                               float& m, float& z, float& v, float& u) {
     if (lim < 0) return;
+    if (m != -INFINITY) {
+        float zs = 0.f, vs = 0.f, us = 0.f;
+        if (lim >= 31)
+            exp_word_both<false>(x, sl2, -m, 31, vm, zs, vs, us);
+        else
+            exp_word_both<true>(x, sl2, -m, lim, vm, zs, vs, us);
+        if (zs <= kWordSumLimit) {
+            z += zs;
+            v += vs;
+            u += us;
+            return;
+        }
+    }
     const float m_new = fmaxf(m, (lim >= 31 ? max32(x) : max32_masked(x, lim)) * sl2);
     const float alpha = fast_exp2(m - m_new);
     z *= alpha;
@@ -132,26 +181,6 @@ __device__ __forceinline__ void row_word_both(const float (&x)[32], float sl2, i
     else
         exp_word_both<true>(x, sl2, -m_new, lim, vm, z, v, u);
     m = m_new;
-}
-
-__device__ __forceinline__ void row_word(const float (&x)[32], float sl2, int lim, uint32_t vm,
-                                         float& m, float& z, float& v) {
-    if (lim < 0) return;
-    if (lim >= 31) {
-        const float m_new = fmaxf(m, max32(x) * sl2);
-        const float alpha = fast_exp2(m - m_new);
-        z *= alpha;
-        v *= alpha;
-        exp_word<false>(x, sl2, -m_new, 31, vm, z, v);
-        m = m_new;
-    } else {
-        const float m_new = fmaxf(m, max32_masked(x, lim) * sl2);
-        const float alpha = fast_exp2(m - m_new);
-        z *= alpha;
-        v *= alpha;
-        exp_word<true>(x, sl2, -m_new, lim, vm, z, v);
-        m = m_new;
-    }
 }
 
 }  // namespace tgvkv
