@@ -6,6 +6,11 @@
 // rows straight away.  The layer budgets come in from global memory (on the
 // evict path the score kernel derives them).
 //
+// In the fused form the rows of the text runs before the first and after the
+// last vision key ("edge" rows) have slots that the budget alone fixes (the
+// first rows and the last rows of the set), so extra CTAs copy them while the
+// selecting CTAs select; a selecting CTA gathers the interior rows only.
+//
 // Selection: the scores become order-preserving 32-bit keys in shared memory;
 // an MSB-first radix select (four 8-bit digits) finds the key T of the b_l-th
 // largest score and how many keys equal to T are still needed (k_eq).  A
@@ -51,6 +56,70 @@ __device__ __forceinline__ int block_exclusive_scan(int x, int* buf, int* total)
     return res;
 }
 
+// First vision position (N if none) and one past the last (0 if none) of the
+// modality bytes in shared memory, reduced over the block.
+__device__ __forceinline__ void vision_span_block(const uint8_t* modality, int N, int* lo, int* hi,
+                                                  int* red) {
+    int a = N, z = 0;
+    for (int j = threadIdx.x; j < N; j += blockDim.x)
+        if (modality[j]) {
+            a = min(a, j);
+            z = max(z, j + 1);
+        }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        a = min(a, __shfl_xor_sync(~0u, a, o));
+        z = max(z, __shfl_xor_sync(~0u, z, o));
+    }
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+    if (lane == 0) {
+        red[warp] = a;
+        red[32 + warp] = z;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        for (int w = 1; w < nw; ++w) {
+            red[0] = min(red[0], red[w]);
+            red[32] = max(red[32], red[32 + w]);
+        }
+    }
+    __syncthreads();
+    *lo = red[0];
+    *hi = red[32];
+    __syncthreads();
+}
+
+// Copy `rows` consecutive K and V rows of head `head` starting at position
+// `src0` to output rows starting at `dst0`, with the threads [t0, t0 + nt)
+// (16-byte vectors, loads before stores).
+template <int VPR>
+__device__ __forceinline__ void copy_rows(const uint4* __restrict__ k, const uint4* __restrict__ v,
+                                          uint4* __restrict__ k_out, uint4* __restrict__ v_out,
+                                          size_t head, int src0, long long dst0, int rows, int t,
+                                          int nt) {
+    constexpr int UNROLL = 4;
+    const int nvec = rows * VPR;
+    for (int i0 = t; i0 < nvec; i0 += nt * UNROLL) {
+        uint4 kr[UNROLL], vr[UNROLL];
+#pragma unroll
+        for (int u = 0; u < UNROLL; ++u) {
+            const int i = i0 + u * nt;
+            if (i < nvec) {
+                kr[u] = __ldg(k + (head + src0) * VPR + i);
+                vr[u] = __ldg(v + (head + src0) * VPR + i);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < UNROLL; ++u) {
+            const int i = i0 + u * nt;
+            if (i < nvec) {
+                k_out[(size_t)dst0 * VPR + i] = kr[u];
+                v_out[(size_t)dst0 * VPR + i] = vr[u];
+            }
+        }
+    }
+}
+
 // Shared memory of one CTA: keys [N_v], retained rows [N] (gather form) and
 // the modality bytes [N].
 __host__ __device__ inline size_t select_smem(const Problem& p, bool compact) {
@@ -77,8 +146,13 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
     __shared__ int s_kk;
     __shared__ long long s_off;
 
-    const int lg = blockIdx.x, l = lg / p.H_kv, g = lg % p.H_kv;
+    // fused form: CTA 2h selects head h and gathers its interior rows, CTA
+    // 2h + 1 copies its edge rows
+    const int lg = COMPACT ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+    const bool edge_cta = COMPACT && (blockIdx.x & 1);
+    const int l = lg / p.H_kv, g = lg % p.H_kv;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    __shared__ int span_red[64];
 
     for (int j = tid; j < p.N; j += kThreads) modality[j] = __ldg(modality_g + j);
     int b = budgets[l];
@@ -100,6 +174,20 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(~0u, part, o);
         if (lane == 0) off_part[warp] = part;
+    }
+    __syncthreads();
+    int vlo = 0, vhi = 0;   // edge rows: positions [0, vlo) and [vhi, N)
+    if (COMPACT) vision_span_block(modality, p.N, &vlo, &vhi, span_red);
+    if (vhi < vlo) vhi = vlo;   // no vision key: every row is a leading edge row
+    if (edge_cta) {
+        long long off = (long long)g * len;
+        for (int w = 0; w < kThreads / 32; ++w) off += off_part[w];
+        const size_t head = (size_t)lg * p.N;
+        const int tail = p.N - vhi;
+        if (vlo <= len) copy_rows<VPR>(k, v, k_out, v_out, head, 0, off, vlo, tid, kThreads);
+        if (tail <= len - vlo)
+            copy_rows<VPR>(k, v, k_out, v_out, head, vhi, off + len - tail, tail, tid, kThreads);
+        return;
     }
     const float* sc = scores + (size_t)lg * p.N_v;
     for (int i = tid; i < p.N_v; i += kThreads) keys[i] = float_order_key(__ldg(sc + i));
@@ -218,14 +306,17 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
     if (tid == 0 && tot != len) raise_status(status, TGVKV_STATUS_COUNT);
     if (!COMPACT) return;
 
-    // ---- gather the retained K and V rows (fused form)
+    // ---- gather the interior retained K and V rows (fused form): the set's
+    // first vlo rows and last N - vhi rows are the edge CTA's
     __syncthreads();
     constexpr int RPI = 32 / VPR;     // rows per warp per step
     constexpr int UNROLL = 4;
-    const int n = min(len, tot);
+    const bool edges_ok = vlo <= len && p.N - vhi <= len - vlo;
+    const int n = min(len, tot) - (edges_ok ? p.N - vhi : 0);
+    const int rfirst = edges_ok ? vlo : 0;
     const int sub = lane / VPR, vec = lane % VPR;
     const size_t head = (size_t)lg * p.N;
-    for (int r0 = warp * RPI * UNROLL; r0 < n; r0 += (kThreads / 32) * RPI * UNROLL) {
+    for (int r0 = rfirst + warp * RPI * UNROLL; r0 < n; r0 += (kThreads / 32) * RPI * UNROLL) {
         uint4 kr[UNROLL], vr[UNROLL];
 #pragma unroll
         for (int u = 0; u < UNROLL; ++u) {
@@ -275,7 +366,14 @@ tpr_select_warp_kernel(Problem p, const float* __restrict__ scores,
     int* rows = hist + 256;
     for (int j = threadIdx.x; j < p.N; j += blockDim.x) modality[j] = __ldg(modality_g + j);
     __syncthreads();
-    const int lg = blockIdx.x * nw + wid;
+    // CTA 2c selects and gathers the interior rows of heads c*nw.., CTA 2c + 1
+    // copies their edge rows (positions [0, vlo) and [vhi, N))
+    __shared__ int span_red[64];
+    int vlo, vhi;
+    vision_span_block(modality, p.N, &vlo, &vhi, span_red);
+    if (vhi < vlo) vhi = vlo;
+    const bool edge_cta = blockIdx.x & 1;
+    const int lg = (int)(blockIdx.x >> 1) * nw + wid;
     if (lg >= p.L * p.H_kv) return;
     const int l = lg / p.H_kv, g = lg % p.H_kv;
     const uint32_t lt = (1u << lane) - 1u;
@@ -296,6 +394,16 @@ tpr_select_warp_kernel(Problem p, const float* __restrict__ scores,
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) off += __shfl_xor_sync(~0u, off, o);
     off += (long long)g * len;
+    const int tail = p.N - vhi;
+    const bool edges_ok = vlo <= len && tail <= len - vlo;
+    if (edge_cta) {
+        if (edges_ok) {
+            const size_t head = (size_t)lg * p.N;
+            copy_rows<VPR>(k, v, k_out, v_out, head, 0, off, vlo, lane, 32);
+            copy_rows<VPR>(k, v, k_out, v_out, head, vhi, off + len - tail, tail, lane, 32);
+        }
+        return;
+    }
     if (lane == 0) {
         offsets[lg] = off;
         if (lg == p.L * p.H_kv - 1) offsets[lg + 1] = off + len;
@@ -388,13 +496,14 @@ tpr_select_warp_kernel(Problem p, const float* __restrict__ scores,
     if (lane == 0 && out_base != len) raise_status(status, TGVKV_STATUS_COUNT);
     __syncwarp();
 
-    // ---- gather the retained K and V rows
+    // ---- gather the interior retained K and V rows (the edge CTA copies the rest)
     constexpr int RPI = 32 / VPR;   // rows per warp instruction
     constexpr int UNROLL = 8;
-    const int n = min(len, out_base);
+    const int n = min(len, out_base) - (edges_ok ? tail : 0);
+    const int rfirst = edges_ok ? vlo : 0;
     const int sub = lane / VPR, vec = lane % VPR;
     const size_t head = (size_t)lg * p.N;
-    for (int r0 = 0; r0 < n; r0 += RPI * UNROLL) {
+    for (int r0 = rfirst; r0 < n; r0 += RPI * UNROLL) {
         uint4 kr[UNROLL], vr[UNROLL];
 #pragma unroll
         for (int u = 0; u < UNROLL; ++u) {
@@ -735,7 +844,7 @@ cudaError_t launch_sel_warp(const Problem& p, int nw, const float* scores, const
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const int heads = p.L * p.H_kv;
-    kern<<<(heads + nw - 1) / nw, nw * 32, smem, stream>>>(
+    kern<<<2 * ((heads + nw - 1) / nw), nw * 32, smem, stream>>>(
         p, scores, budgets, modality, offsets, idx, reinterpret_cast<const uint4*>(k),
         reinterpret_cast<const uint4*>(v), reinterpret_cast<uint4*>(k_out),
         reinterpret_cast<uint4*>(v_out), status);
@@ -751,7 +860,7 @@ cudaError_t launch_sel(const Problem& p, const float* scores, const int32_t* bud
     const size_t smem = select_smem(p, COMPACT);
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    kern<<<p.L * p.H_kv, kThreads, smem, stream>>>(
+    kern<<<p.L * p.H_kv * (COMPACT ? 2 : 1), kThreads, smem, stream>>>(
         p, scores, budgets, modality, offsets, idx,
         reinterpret_cast<const uint4*>(k),
         reinterpret_cast<const uint4*>(v), reinterpret_cast<uint4*>(k_out),
