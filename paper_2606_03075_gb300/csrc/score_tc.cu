@@ -209,11 +209,12 @@ __device__ __forceinline__ bool next_step(const Item& it, int mode, int pass, in
 }
 
 // Sum over the valid rows of one 32-row group of 2^(y_i sl2 + nmp_i), with the
-// causal mask j <= pos_i unless every row sees key j.  FULL: all 32 rows exist.
-template <bool FULL>
+// causal mask j <= pos_i.  FULL: all 32 rows exist; ALL_VIS: every row sees
+// key j (no mask; a template argument, so that the unrolled loop has no
+// branch on it).
+template <bool FULL, bool ALL_VIS>
 __device__ __forceinline__ float colsum_group(const float (&y)[32], const float* nmp,
-                                              const int* pos, float sl2, int rpg, int j,
-                                              bool all_vis) {
+                                              const int* pos, float sl2, int rpg, int j) {
     const float2 s2 = make_float2(sl2, sl2);
     float2 a = make_float2(0.f, 0.f), b = a;
 #pragma unroll
@@ -224,7 +225,7 @@ __device__ __forceinline__ float colsum_group(const float (&y)[32], const float*
             const float2 t1 = fma2(make_float2(y[i + 2], y[i + 3]), s2, make_float2(n4.z, n4.w));
             float2 e0 = make_float2(fast_exp2(t0.x), fast_exp2(t0.y));
             float2 e1 = make_float2(fast_exp2(t1.x), fast_exp2(t1.y));
-            if (!all_vis) {
+            if (!ALL_VIS) {
                 const int4 p4 = *reinterpret_cast<const int4*>(pos + i);
                 if (j > p4.x) e0.x = 0.f;
                 if (j > p4.y) e0.y = 0.f;
@@ -852,10 +853,17 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
                             if (ch == nch - 1) release_acc(&s.s_empty[b], lane);
                             const float* nmp = s.row_nmp[rs] + rcol + ch * 32;
                             const int* rp = s.row_pos[rs] + rcol + ch * 32;
-                            if (rpg >= 32)
-                                sum += colsum_group<true>(y, nmp, rp, sl2, rpg, j, all_vis);
-                            else
-                                sum += colsum_group<false>(y, nmp, rp, sl2, rpg, j, all_vis);
+                            if (rpg >= 32) {
+                                if (all_vis)
+                                    sum += colsum_group<true, true>(y, nmp, rp, sl2, rpg, j);
+                                else
+                                    sum += colsum_group<true, false>(y, nmp, rp, sl2, rpg, j);
+                            } else {
+                                if (all_vis)
+                                    sum += colsum_group<false, true>(y, nmp, rp, sl2, rpg, j);
+                                else
+                                    sum += colsum_group<false, false>(y, nmp, rp, sl2, rpg, j);
+                            }
                         }
                     }
                     if (ok && act) {
