@@ -93,7 +93,7 @@ extern "C" {
 #define TGVKV_STATUS_TEXT_POS     0x01u /* text_pos not strictly ascending or outside [0, N) */
 #define TGVKV_STATUS_VISION_COUNT 0x02u /* modality marks a vision count other than N_v */
 #define TGVKV_STATUS_BUDGET       0x04u /* a layer budget outside [0, N_v] reached select */
-#define TGVKV_STATUS_INDEX        0x08u /* compact: an index outside [0, N), or a CSR larger than the output */
+#define TGVKV_STATUS_INDEX        0x08u /* compact: an index outside [0, N), or a CSR larger than the output; decode: a CSR outside its rows */
 #define TGVKV_STATUS_COUNT        0x10u /* a retained set did not hold N_t + b_l rows */
 #define TGVKV_STATUS_TIMEOUT      0x20u /* a bounded on-chip wait gave up */
 #define TGVKV_STATUS_WEIGHT       0x40u /* a text weight is negative or not finite */
@@ -300,18 +300,25 @@ int tgvkv_evict_launches(const tgvkv_desc* desc);
  * layer l attends to the rows of set (l, g = h / G) of a CSR cache:
  *   out[l][h][:] = sum_r softmax_r(softmax_scale * <q[l][h], k_rows[r]>) v_rows[r]
  * over r in [offsets[l*H_kv+g], offsets[l*H_kv+g+1]); an empty set gives 0.
- * q: bf16 [L][H_q][d]; k_rows, v_rows: bf16 [rows][d] (k_out / v_out of
- * tgvkv_evict, or the full cache [L][H_kv][N][d] with offsets[i] = i * N);
- * offsets: int64 [L*H_kv + 1]; out: fp32 [L][H_q][d] (output).  bf16 products,
- * fp32 accumulation and softmax.  The workspace holds the row-split partials
- * (tgvkv_workspace_size covers them). */
+ * q: bf16 [L][H_q][d], 16-byte aligned; k_rows, v_rows: bf16 [rows][d], 16-byte
+ * aligned (k_out / v_out of tgvkv_evict, or the full cache [L][H_kv][N][d]
+ * with offsets[i] = i * N), each holding at least capacity_rows rows;
+ * offsets: int64 [L*H_kv + 1], nondecreasing; out: fp32 [L][H_q][d] (output),
+ * 8-byte aligned.  bf16 products, fp32 accumulation and softmax; the softmax
+ * weights enter the value sum as bf16(P) + bf16(P - bf16(P)) (about 16 bits).
+ * Rows at or above capacity_rows (and above 2^31 - 1) are never read: a set
+ * that reaches them, or a decreasing or negative offset, sets
+ * TGVKV_STATUS_INDEX (results then undefined).  capacity_rows < 0 is
+ * rejected.  The rows of other sets
+ * next to a set's own may be read and are masked: they must be finite.
+ * Two kernels: the row streams, then (launched as a programmatic dependent)
+ * the merge of the sets they split; the workspace holds the streams' partial
+ * results (tgvkv_workspace_size covers them). */
 int tgvkv_decode(const tgvkv_desc* desc, const uint16_t* q, const uint16_t* k_rows,
-                 const uint16_t* v_rows, const int64_t* offsets, float* out,
-                 void* workspace, void* stream);
+                 const uint16_t* v_rows, int64_t capacity_rows, const int64_t* offsets,
+                 float* out, void* workspace, void* stream);
 
-/* Kernels one tgvkv_decode call launches (1, or 2 when few KV heads make it
- * split each set's rows over several CTAs and merge them).  -1 on bad
- * arguments. */
+/* Kernels one tgvkv_decode call launches (2).  -1 on bad arguments. */
 int tgvkv_decode_launches(const tgvkv_desc* desc);
 
 /* Zero `workspace` (asynchronously on `stream`).  Needed once after the
@@ -350,9 +357,10 @@ const char* tgvkv_last_error(void);
  * library holds that array until the process exits.  Nothing is allocated.
  *
  * Same arguments and results as tgvkv_score, minus the workspace.
- * - A problem whose scratch exceeds TGVKV_NOALLOC_SCRATCH_BYTES (see
- *   tgvkv_workspace_size) is rejected with TGVKV_ERR_UNSUPPORTED before any
- *   launch.
+ * - A problem whose scratch (the part of the tgvkv_workspace_size workspace
+ *   that tgvkv_score uses: all of it but the decode partials at its end)
+ *   exceeds TGVKV_NOALLOC_SCRATCH_BYTES is rejected with
+ *   TGVKV_ERR_UNSUPPORTED before any launch.
  * - Every call looks up the array's device address in the current device's
  *   context (so a context created after cudaDeviceReset uses its own array);
  *   the first call on a device may load the library's device code, so make it

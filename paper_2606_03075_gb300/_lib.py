@@ -60,8 +60,8 @@ SIGNATURES = {
     "tgvkv_workspace_init": (c_int, [_P, c_void_p, c_void_p]),
     "tgvkv_status": (c_int, [c_void_p, c_void_p]),
     "tgvkv_evict_launches": (c_int, [_P]),
-    "tgvkv_decode": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
-                             c_void_p]),
+    "tgvkv_decode": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_int64, c_void_p, c_void_p,
+                             c_void_p, c_void_p]),
     "tgvkv_decode_launches": (c_int, [_P]),
     "tgvkv_check_wait_timeout": (c_int, [c_void_p, c_void_p]),
     "tgvkv_last_error": (c_char_p, []),

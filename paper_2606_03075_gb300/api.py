@@ -325,11 +325,13 @@ def tgvkv_status(ws: torch.Tensor, stream=None) -> int:
 def tgvkv_decode(desc, q, k_rows, v_rows, offsets, out, ws, stream=None):
     """One decode step of every layer over a CSR cache (see include/tgvkv.h)."""
     L, Hq, Hkv, d = desc.L, desc.H_q, desc.H_kv, desc.d
+    capacity = min(k_rows.numel(), v_rows.numel()) // d
     _check(_lib.load().tgvkv_decode(
         ctypes.byref(desc),
         _ptr(q, _BF16_LIKE, L * Hq * d, "q"),
         _ptr(k_rows, _BF16_LIKE, 0, "k_rows"),
         _ptr(v_rows, _BF16_LIKE, 0, "v_rows"),
+        capacity,
         _ptr(offsets, (torch.int64,), L * Hkv + 1, "offsets"),
         _ptr(out, (torch.float32,), L * Hq * d, "out"),
         _ptr(ws, (torch.uint8,), tgvkv_workspace_size(desc), "workspace"),

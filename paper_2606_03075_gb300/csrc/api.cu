@@ -54,15 +54,17 @@ WsLayout layout_of(const Problem& p) {
     const size_t keyset = (size_t)(p.N_v > p.N_t ? p.N_v : p.N_t);
     if (p.T > 1) o += round_up(sizeof(float) * (size_t)p.L * p.H_kv * p.T * keyset);
     w.stat_text = o;   o += round_up(sizeof(float) * (size_t)p.L);
-    w.decode_part = o;
-    if (decode_splits(p) > 1)
-        o += round_up(sizeof(float) * (size_t)p.L * p.H_q * decode_splits(p) * (p.d + 2));
     w.text_scores = w.weights = w.row_stats = 0;
     if (needs_text_pass(p)) {
         w.text_scores = o; o += round_up(sizeof(float) * (size_t)p.L * p.H_kv * (p.N_t > 0 ? p.N_t : 1));
         w.weights = o;     o += round_up(sizeof(float) * (size_t)p.L * (p.n_win > 0 ? p.n_win : 1));
         w.row_stats = o;   o += round_up(3 * sizeof(float) * ((size_t)p.L * p.H_q * p.n_win + 1));
     }
+    w.score_total = o;
+    // decode only, after everything the score and eviction calls use
+    w.decode_part = o;
+    o += round_up(sizeof(float) * (size_t)decode_passes(p) * kDecMaxStreams * 2 *
+                  decode_record_floats(p));
     w.total = o;
     return w;
 }
@@ -494,21 +496,28 @@ int tgvkv_prefill(const tgvkv_desc* desc, const uint16_t* q, const uint16_t* k, 
 }
 
 int tgvkv_decode(const tgvkv_desc* desc, const uint16_t* q, const uint16_t* k_rows,
-                 const uint16_t* v_rows, const int64_t* offsets, float* out, void* workspace,
-                 void* stream) {
+                 const uint16_t* v_rows, int64_t capacity_rows, const int64_t* offsets,
+                 float* out, void* workspace, void* stream) {
     Problem p{};
     int rc = make_problem(desc, &p);
     if (rc) return rc;
-    REQUIRE_PTR(q, "q", false);
+    REQUIRE_PTR(q, "q", true);
     REQUIRE_PTR(k_rows, "k_rows", true);
     REQUIRE_PTR(v_rows, "v_rows", true);
     REQUIRE_PTR(offsets, "offsets", false);
     REQUIRE_PTR(out, "out", false);
     REQUIRE_PTR(workspace, "workspace", true);
+    if (capacity_rows < 0)
+        return fail(TGVKV_ERR_INVALID_ARG, "capacity_rows=%lld < 0", (long long)capacity_rows);
+    if ((reinterpret_cast<uintptr_t>(offsets) & 7u) != 0)
+        return fail(TGVKV_ERR_INVALID_ARG, "offsets is not 8-byte aligned");
+    if ((reinterpret_cast<uintptr_t>(out) & 7u) != 0)
+        return fail(TGVKV_ERR_INVALID_ARG, "out is not 8-byte aligned");
     const WsLayout lay = layout_of(p);
-    cudaError_t e = launch_decode(p, q, k_rows, v_rows, offsets, out,
-                                  reinterpret_cast<float*>(static_cast<char*>(workspace) + lay.decode_part),
-                                  static_cast<cudaStream_t>(stream));
+    char* ws = static_cast<char*>(workspace);
+    cudaError_t e = launch_decode(p, q, k_rows, v_rows, (long long)capacity_rows, offsets, out,
+                                  reinterpret_cast<float*>(ws + lay.decode_part),
+                                  status_of(workspace, lay), static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? ok() : cuda_fail(e, "decode launch");
 }
 
@@ -599,11 +608,11 @@ extern "C" int tgvkv_score_noalloc(const tgvkv_desc* desc, const uint16_t* q_tex
     int rc = make_problem(desc, &p);
     if (rc) return rc;
     const WsLayout lay = layout_of(p);
-    if (lay.total > (size_t)TGVKV_NOALLOC_SCRATCH_BYTES)
+    if (lay.score_total > (size_t)TGVKV_NOALLOC_SCRATCH_BYTES)
         return fail(TGVKV_ERR_UNSUPPORTED,
                     "problem needs %zu bytes of scratch; the static scratch holds %u "
                     "(use tgvkv_score with a caller workspace)",
-                    lay.total, (unsigned)TGVKV_NOALLOC_SCRATCH_BYTES);
+                    lay.score_total, (unsigned)TGVKV_NOALLOC_SCRATCH_BYTES);
     void* scratch = nullptr;
     if ((rc = noalloc_scratch(&scratch))) return rc;
     rc = check_score_args(p, q_text, k, modality, text_pos, w, scores, tvb_stat, scratch);

@@ -31,15 +31,17 @@ struct Problem {
     int stats_given;
 };
 
-// Row splits of the decode kernel: enough CTAs for two per SM on the 152 SMs
-// of a GB300 when there are few KV heads, at most one split per 128 positions.
-__host__ __device__ inline int decode_splits(const Problem& p) {
-    const int ctas = p.L * p.H_kv * ((p.G + 7) / 8);
-    int s = (2 * 152 + ctas - 1) / ctas;
-    const int most = (p.N + 127) / 128;
-    if (s > most) s = most;
-    if (s > 16) s = 16;
-    return s < 1 ? 1 : s;
+// Decode (decode.cu): at most kDecMaxStreams row streams (warps; one CTA per
+// SM); a stream leaves at most two partial results of decode_heads(p) query
+// heads x (d + 2) floats per pass over the rows, a pass taking up to 8 query
+// heads of a group.
+constexpr int kDecMaxStreams = 2048;
+__host__ __device__ inline int decode_passes(const Problem& p) { return (p.G + 7) / 8; }
+__host__ __device__ inline int decode_heads(const Problem& p) { return p.G < 8 ? p.G : 8; }
+// floats of one partial result: O [heads][d], then m [heads] and l [heads],
+// padded to a multiple of 4 floats (16-byte aligned records)
+__host__ __device__ inline int decode_record_floats(const Problem& p) {
+    return decode_heads(p) * p.d + ((2 * decode_heads(p) + 3) & ~3);
 }
 
 // Sinks among the positions 0..N-1: the first keep_first and the last keep_last.
@@ -59,7 +61,9 @@ struct WsLayout {
     size_t weights;     // float [L*n_win]: Eq. 7 weights
     size_t stat_text;   // float [L]: the text-key pass's (unused) statistic
     size_t row_stats;   // float [3*L*H_q*n_win]: per-row (m, Z, vision mass) of the text-key pass
-    size_t decode_part; // float [L*H_q*S*(d+2)]: decode row-split partials (S > 1)
+    size_t score_total; // bytes of everything above: what tgvkv_score / tgvkv_evict use
+    // tgvkv_decode only (after score_total):
+    size_t decode_part; // float [passes*kDecMaxStreams*2*record]: partials of split sets
     size_t total;
 };
 

@@ -46,10 +46,12 @@ cudaError_t launch_eq7_weights(const Problem& p, const float* text_scores, const
                                const int32_t* text_pos, float* weights, uint32_t* status,
                                cudaStream_t stream);
 
-// Decode over the compacted cache (decode.cu): out[l][h][:] for one new token.
+// Decode over the compacted cache (decode.cu): out[l][h][:] for one new token
+// (two kernels: the row streams, then the merge of the sets they split).  Rows
+// from capacity_rows on are never read.
 cudaError_t launch_decode(const Problem& p, const uint16_t* q, const uint16_t* k_rows,
-                          const uint16_t* v_rows, const int64_t* offsets, float* out, float* part,
-                          cudaStream_t stream);
+                          const uint16_t* v_rows, long long capacity_rows, const int64_t* offsets,
+                          float* out, float* part, uint32_t* status, cudaStream_t stream);
 int decode_launches(const Problem& p);
 
 // Kernels launch_score / launch_select_compact launch for p.

@@ -329,6 +329,63 @@ def test_decode_empty_sets_give_zero(api):
     assert np.array_equal(o, np.zeros_like(o))
 
 
+# Ragged CSR layouts around the decode kernel's boxes (8 and 32 rows): sets of
+# 0, 1, 7-9, 15-17, 31-33, 63-65 and 257 rows, empty sets between full ones, a
+# base offset before the first set and spare rows after the last; groups of 1,
+# 4 and 12 query heads (12 takes two passes of 8 heads) at d = 64 and 128; and
+# one long set that every row stream of the GPU shares (merged from all of
+# their partial results).
+_RAGGED_LENS = [0, 1, 7, 8, 9, 15, 16, 17, 31, 32, 33, 0, 63, 64, 65, 257, 0, 3]
+
+
+def _ragged_decode(api, L, H_kv, G, d, lens, base, spare, seed):
+    wl = synth.custom("ragged", L, G * H_kv, H_kv, d, [("text", 8), ("vision", 300), ("text", 8)])
+    desc = api.desc_for_workload(wl)
+    rng = np.random.default_rng(seed)
+    offsets = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64) + base
+    n_rows = int(offsets[-1]) + spare
+    k_bits = synth.to_bf16_bits(rng.standard_normal((n_rows, d)).astype(np.float32))
+    v_bits = synth.to_bf16_bits(rng.standard_normal((n_rows, d)).astype(np.float32))
+    qb = _decode_q(wl, seed + 1)
+    dev = lambda b: torch.from_numpy(np.ascontiguousarray(b)).cuda().view(torch.bfloat16)
+    off_d = torch.from_numpy(offsets).cuda()
+    o = _run_decode(api, desc, qb, dev(k_bits), dev(v_bits), off_d)
+    ref = _oracle_decode(wl, qb, k_bits, v_bits, offsets)
+    return o, ref
+
+
+@pytest.mark.parametrize("d", [64, 128])
+@pytest.mark.parametrize("G", [1, 4, 12])
+def test_decode_ragged_csr(api, d, G):
+    """Decode over ragged CSR layouts, element by element against the oracle."""
+    L, H_kv = 3, 6
+    lens = _RAGGED_LENS
+    o, ref = _ragged_decode(api, L, H_kv, G, d, lens, base=5, spare=37, seed=20 + G + d)
+    P.assert_close(o, ref, f"decode, ragged CSR (G={G}, d={d})", floor=DEC_FLOOR)
+
+
+@pytest.mark.parametrize("G", [1, 7])
+def test_decode_one_long_set(api, G):
+    """One set of 40 000 rows: every row stream takes a slice of it, and the last
+    stream to finish merges all partial results."""
+    o, ref = _ragged_decode(api, 1, 1, G, 128, [40000], base=0, spare=0, seed=31 + G)
+    P.assert_close(o, ref, f"decode, one long set (G={G})", floor=DEC_FLOOR)
+
+
+def test_decode_csr_past_capacity(api):
+    """A CSR whose last set runs past the rows the buffers hold: the kernel
+    reads no row from capacity_rows on and reports TGVKV_STATUS_INDEX."""
+    wl = synth.custom("short_cache", 1, 4, 2, 128, [("text", 8), ("vision", 300), ("text", 8)])
+    desc = api.desc_for_workload(wl)
+    rows = torch.zeros((100, wl.d), dtype=torch.bfloat16, device="cuda")
+    offsets = torch.tensor([0, 60, 180], dtype=torch.int64, device="cuda")
+    ws = api.new_workspace(desc)
+    out = torch.empty((desc.L, desc.H_q, desc.d), dtype=torch.float32, device="cuda")
+    qd = torch.from_numpy(_decode_q(wl, 3)).cuda().view(torch.bfloat16)
+    api.tgvkv_decode(desc, qd, rows, rows, offsets, out, ws)
+    assert api.tgvkv_status(ws) == 0x08
+
+
 # ---------------------------------------------------------------- layer-budget statistics (Table 1a)
 @pytest.mark.parametrize("name", ["mha_single", "gqa_pairs", "text_heavy"])
 @pytest.mark.parametrize("stat", ["tt", "uniform"])

@@ -47,7 +47,6 @@ def test_noalloc_matches_workspace_call(wl):
     inp = synth.generate(wl, seed=7)
     dev = P.device_inputs(inp)
     desc = api.desc_for_workload(wl)
-    assert api.tgvkv_workspace_size(desc) <= 8 << 20
     stream = torch.cuda.current_stream()
 
     ws = api.new_workspace(desc)
