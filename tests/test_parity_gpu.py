@@ -52,8 +52,9 @@ SMALL = {
 }
 
 
-# Heads of one row tile with 64 < G * n_win <= 128 and d = 128 (the score
-# kernel's single-tile items) at several lengths, row counts and causal layouts.
+# Heads of one row tile with 64 < G * n_win <= 128 (the score kernel's
+# single-tile items) at several lengths, row counts, causal layouts and head
+# dims.
 ONE_TILE = {
     # grouped-query heads (G = 2, 96 rows)
     "gqa_96": synth.custom("gqa_96", 2, 8, 4, 128,
@@ -82,6 +83,16 @@ ONE_TILE = {
     "long_r128": synth.custom("long_r128", 1, 4, 2, 128,
                              [("text", 17), ("vision", 2800), ("text", 64)], window=64,
                              ratios=(0.05,)),
+    # one KV head in all
+    "one_head_96": synth.custom("one_head_96", 1, 1, 1, 128,
+                                [("text", 12), ("vision", 600), ("text", 96)], ratios=(0.1,)),
+    # one key tile per head
+    "one_key_tile_96": synth.custom("one_key_tile_96", 2, 2, 2, 128,
+                                    [("text", 4), ("vision", 20), ("text", 96)], ratios=(0.25,)),
+    # d = 64, an odd number of key tiles
+    "d64_96": synth.custom("d64_96", 3, 4, 4, 64,
+                           [("text", 9), ("vision", 500), ("text", 25), ("vision", 70),
+                            ("text", 96)], ratios=(0.1,)),
 }
 
 
