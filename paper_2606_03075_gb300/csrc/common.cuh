@@ -84,6 +84,18 @@ constexpr int kMaxN = 32768;     // key positions per head (the per-CTA tile map
 constexpr int kMaxNv = 49152;    // vision keys held in shared memory by select
 constexpr int kMaxL = 1024;      // layers handled by the budget kernel
 
+// Programmatic dependent launch: a kernel launched with the programmatic
+// stream-serialization attribute may start while the kernel before it on the
+// stream runs; griddep_wait blocks until that kernel has completed (a no-op
+// for an ordinary launch).  What that kernel wrote must then be read through
+// L2 (__ldcg), not the read-only path: a dependent that started early can
+// otherwise read a recycled buffer's old contents.  A kernel that calls
+// griddep_launch_dependents lets its dependent be scheduled from then on.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 __device__ __forceinline__ void raise_status(uint32_t* status, uint32_t bits) {
     atomicOr(status, bits);
 }

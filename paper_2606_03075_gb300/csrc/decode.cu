@@ -225,7 +225,7 @@ decode_kernel(const __grid_constant__ CUtensorMap mkf, const __grid_constant__ C
               float* __restrict__ part, uint32_t* __restrict__ status) {
     using Gm = DecGeom<D, CH, W>;
     // the merge kernel may be scheduled now; it waits for this grid's results
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    griddep_launch_dependents();
     if (threadIdx.x == 0) {   // the descriptors' first fetch overlaps the prologue
         tc::tma_prefetch_desc(&mkf);
         tc::tma_prefetch_desc(&mk8);
@@ -497,6 +497,8 @@ decode_merge_kernel(const Problem p, const int64_t* __restrict__ offsets, int ca
     const int hpp = decode_heads(p), rec = decode_record_floats(p);
     const int gw = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
     const int s = gw / hpp, hh = gw % hpp;
+    // inputs only before the wait (the first kernel writes none of them); its
+    // partial results after it, through L2
     long long lo_raw = 0, hi_raw = 0, r0_raw = 0, r1_raw = 0;
     if (s < n_sets) {
         lo_raw = offsets[s];
@@ -504,7 +506,7 @@ decode_merge_kernel(const Problem p, const int64_t* __restrict__ offsets, int ca
         r0_raw = offsets[0];
         r1_raw = offsets[n_sets];
     }
-    asm volatile("griddepcontrol.wait;" ::: "memory");
+    griddep_wait();
     if (s >= n_sets || hh >= nh) return;
     // every set's rows must lie in order inside [0, cap)
     if (hh == 0 && lane == 0 && (lo_raw < 0 || hi_raw < lo_raw || hi_raw > cap))
@@ -630,19 +632,10 @@ cudaError_t launch_dec(const Problem& p, const uint16_t* q, const uint16_t* k_ro
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     // the merge, as a programmatic dependent: it is scheduled while the first
     // kernel runs and waits on the device for its results
-    cudaLaunchConfig_t cfg = {};
     const long long warps = (long long)n_sets * decode_heads(p);
-    cfg.gridDim = dim3((unsigned)((warps + 3) / 4), decode_passes(p));
-    cfg.blockDim = dim3(128);
-    cfg.dynamicSmemBytes = 0;
-    cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, decode_merge_kernel<D>, p, offsets, cap, ctas * W,
-                              static_cast<const float*>(part), out, status);
+    return launch_dependent(decode_merge_kernel<D>, dim3((unsigned)((warps + 3) / 4), decode_passes(p)),
+                            dim3(128), 0, stream, p, offsets, cap, ctas * W,
+                            static_cast<const float*>(part), out, status);
 }
 
 }  // namespace

@@ -11,6 +11,25 @@
 
 namespace tgvkv {
 
+// Launch `kern` as a programmatic dependent of the kernel before it on
+// `stream` (see griddep_wait): its CTAs may be scheduled while that kernel
+// finishes, and must call griddep_wait before reading what it wrote.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_dependent(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                             cudaStream_t stream, Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, static_cast<Args&&>(args)...);
+}
+
 // TWR scores + TVB statistic (score_tc.cu).  The completion counters in the
 // workspace must be zero on entry; the kernel leaves them zero.  When
 // `budgets` is not null, the CTA that finishes last also splits
