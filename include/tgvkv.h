@@ -93,7 +93,7 @@ extern "C" {
 #define TGVKV_STATUS_TEXT_POS     0x01u /* text_pos not strictly ascending or outside [0, N) */
 #define TGVKV_STATUS_VISION_COUNT 0x02u /* modality marks a vision count other than N_v */
 #define TGVKV_STATUS_BUDGET       0x04u /* a layer budget outside [0, N_v] reached select */
-#define TGVKV_STATUS_INDEX        0x08u /* compact: an index outside [0, N), or a CSR larger than the output; decode: a CSR outside its rows */
+#define TGVKV_STATUS_INDEX        0x08u /* compact: an index outside [0, N), decreasing offsets, or a CSR larger than the output; decode: a CSR outside its rows */
 #define TGVKV_STATUS_COUNT        0x10u /* a retained set did not hold N_t + b_l rows */
 #define TGVKV_STATUS_TIMEOUT      0x20u /* a bounded on-chip wait gave up */
 #define TGVKV_STATUS_WEIGHT       0x40u /* a text weight is negative or not finite */

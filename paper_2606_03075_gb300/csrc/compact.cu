@@ -28,6 +28,9 @@ compact_kernel(Problem p, const uint4* __restrict__ k, const uint4* __restrict__
         if (blockIdx.x == 0 && threadIdx.x == 0) raise_status(status, TGVKV_STATUS_INDEX);
         total = total < 0 ? 0 : capacity;
     }
+    // the sets must lie in order (every access below stays in bounds either way)
+    for (int i = blockIdx.x * kThreads + threadIdx.x; i < n_heads; i += gridDim.x * kThreads)
+        if (offsets[i + 1] < offsets[i]) raise_status(status, TGVKV_STATUS_INDEX);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const long long r0 = (long long)blockIdx.x * ROWS_PER_CTA + (long long)warp * ROWS_PER_WARP;
     if (r0 >= total) return;

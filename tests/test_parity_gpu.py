@@ -365,6 +365,27 @@ def test_compact_csr_larger_than_output(api):
     assert not ko[cap:].any() and not vo[cap:].any()
 
 
+def test_compact_decreasing_offsets(api):
+    """Offsets that decrease: TGVKV_STATUS_INDEX, and no row written past the
+    output (every access of the kernel stays in bounds)."""
+    rng = np.random.default_rng(6)
+    L, H, n, d = 2, 2, 40, 128
+    k = rng.integers(-2 ** 15, 2 ** 15, (L, H, n, d)).astype(np.int16)
+    v = rng.integers(-2 ** 15, 2 ** 15, (L, H, n, d)).astype(np.int16)
+    off = np.array([0, 20, 10, 35, 50], np.int64)   # set 1 ends before it starts
+    idx = rng.integers(0, n, 50).astype(np.int32)
+    desc = api.make_desc(L, H, H, d, n, 0, 1)
+    ws = api.new_workspace(desc)
+    cap, guard = 50, 32
+    ko = torch.zeros((cap + guard, d), dtype=torch.int16, device="cuda")
+    vo = torch.zeros((cap + guard, d), dtype=torch.int16, device="cuda")
+    api.tgvkv_compact(desc, torch.from_numpy(k).cuda(), torch.from_numpy(v).cuda(),
+                      torch.from_numpy(off).cuda(), torch.from_numpy(idx).cuda(), ko[:cap], vo[:cap],
+                      ws)
+    assert api.tgvkv_status(ws) & 0x08
+    assert not ko[cap:].any() and not vo[cap:].any()
+
+
 # ---------------------------------------------------------------- full sizes
 FULL = [("llava15", 0.05, (0, 31)), ("llava15", 0.20, (17,)), ("next", 0.05, (0, 31)),
         ("next", 0.10, (5,)), ("next", 0.20, (26,)), ("qwen25", 0.05, (13,)),
