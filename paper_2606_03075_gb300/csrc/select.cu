@@ -15,9 +15,12 @@
 // an MSB-first radix select (four 8-bit digits) finds the key T of the b_l-th
 // largest score and how many keys equal to T are still needed (k_eq).  A
 // vision key is kept iff key > T, or key == T and it is among the first k_eq
-// such keys in position order.  Each thread then owns a contiguous range of
-// positions; three block prefix sums (vision keys, keys equal to T, kept
-// positions) give every kept position its output slot.
+// such keys in position order.  When every key equal to T is kept (the last
+// round's bin holds exactly k_eq keys, the usual case), keep = key >= T and
+// each warp walks a contiguous range of positions with ballots, two block
+// prefix sums giving the ranges their vision rank and output slot bases;
+// with ties to break, each thread owns a range and three block prefix sums
+// (vision keys, keys equal to T, kept positions) give the slots.
 #include "common.cuh"
 #include "launch.h"
 
@@ -128,8 +131,9 @@ __host__ __device__ inline size_t select_smem(const Problem& p, bool compact) {
 }
 
 // COMPACT: also gather the retained rows.
+// (Register bounds: five CTAs per SM in the fused form, eight in the select-only form.)
 template <bool COMPACT, int VPR>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, COMPACT ? 5 : 8)
 tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __restrict__ budgets,
                   const uint8_t* __restrict__ modality_g, int64_t* __restrict__ offsets,
                   int32_t* __restrict__ idx, const uint4* __restrict__ k,
@@ -144,6 +148,7 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
     __shared__ int scan_buf[33];
     __shared__ uint32_t s_prefix;
     __shared__ int s_kk;
+    __shared__ int s_ties;
     __shared__ long long s_off;
 
     // fused form: CTA 2h selects head h and gathers its interior rows, CTA
@@ -236,6 +241,7 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
                         if (kk <= a + cnt[e]) {
                             s_prefix = prefix | ((uint32_t)(255 - 8 * lane - e) << shift);
                             s_kk = kk - a;
+                            s_ties = cnt[e];   // after the last round: the keys equal to T
                             break;
                         }
                         a += cnt[e];
@@ -250,58 +256,103 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
     const bool none = (b == 0);
     const uint32_t thr = prefix;
     const int k_eq = none ? 0 : kk;
-
-    // ---- ordered emission over per-thread position ranges
-    const int per = (p.N + kThreads - 1) / kThreads;
-    const int j0 = min(p.N, tid * per), j1 = min(p.N, j0 + per);
-    int nv = 0;
-    for (int j = j0; j < j1; ++j) nv += modality[j] != 0;
     int tot;
-    const int vbase = block_exclusive_scan(nv, scan_buf, &tot);
-    int neq = 0;
-    if (!none) {
-        int vr = vbase;
-        for (int j = j0; j < j1; ++j)
-            if (modality[j] != 0) {
-                neq += (vr < p.N_v && keys[vr] == thr);
-                ++vr;
-            }
-    }
-    const int ebase = block_exclusive_scan(neq, scan_buf, &tot);
-    // kept(j): text, or a vision key above T, or one of the first k_eq equal to T
-    auto scan_kept = [&](auto&& emit) {
-        int vr = vbase, er = ebase;
-        for (int j = j0; j < j1; ++j) {
-            bool keep = true;
-            if (modality[j] != 0) {
-                keep = false;
-                if (vr < p.N_v && !none) {
-                    const uint32_t key = keys[vr];
-                    if (key > thr) {
-                        keep = true;
-                    } else if (key == thr) {
-                        keep = er < k_eq;
-                        ++er;
-                    }
-                }
-                ++vr;
-            }
-            if (keep) emit(j);
+    long long off;   // read from s_off after a block barrier (with b = 0 no round runs)
+
+    if (none || s_ties == k_eq) {
+        // ---- every key equal to T is kept (no ties to break): a vision key
+        // is kept iff key >= T.  Each warp owns a contiguous range of
+        // positions and walks it 32 at a time with ballots; two block scans
+        // give the ranges their vision rank and output slot bases.
+        const uint32_t lt = (1u << lane) - 1u;
+        constexpr int kWarps = kThreads / 32;
+        const int wper = (((p.N + kWarps - 1) / kWarps) + 31) & ~31;
+        const int w0 = min(p.N, warp * wper), w1 = min(p.N, w0 + wper);
+        int nvw = 0;
+        for (int c0 = w0; c0 < w1; c0 += 32) {
+            const int j = c0 + lane;
+            nvw += __popc(__ballot_sync(~0u, j < w1 && modality[j] != 0));
         }
-    };
-    int nkeep = 0;
-    scan_kept([&](int) { ++nkeep; });
-    const int kbase = block_exclusive_scan(nkeep, scan_buf, &tot);
-    const long long off = s_off;
-    {
-        int r = kbase;
-        scan_kept([&](int j) {
+        const int vbase = __shfl_sync(~0u, block_exclusive_scan(lane == 0 ? nvw : 0, scan_buf, &tot), 0);
+        off = s_off;
+        auto walk = [&](auto&& emit) {
+            int vr = vbase, kr = 0;
+            for (int c0 = w0; c0 < w1; c0 += 32) {
+                const int j = c0 + lane;
+                const bool in = j < w1;
+                const bool isv = in && modality[j] != 0;
+                const uint32_t vb = __ballot_sync(~0u, isv);
+                const int myvr = vr + __popc(vb & lt);
+                const bool keep = in && (!isv || (!none && myvr < p.N_v && keys[myvr] >= thr));
+                const uint32_t kb = __ballot_sync(~0u, keep);
+                if (keep) emit(j, kr + __popc(kb & lt));
+                vr += __popc(vb);
+                kr += __popc(kb);
+            }
+            return kr;
+        };
+        const int nkw = walk([](int, int) {});
+        const int kbase = __shfl_sync(~0u, block_exclusive_scan(lane == 0 ? nkw : 0, scan_buf, &tot), 0);
+        walk([&](int j, int rr) {
+            const int r = kbase + rr;
             if (r < len) {
                 idx[off + r] = j;
                 if (COMPACT) rows[r] = j;
             }
-            ++r;
         });
+    } else {
+        // ---- ties at T to break: ordered emission over per-thread position
+        // ranges, the first k_eq keys equal to T (in position order) kept
+        const int per = (p.N + kThreads - 1) / kThreads;
+        const int j0 = min(p.N, tid * per), j1 = min(p.N, j0 + per);
+        int nv = 0;
+        for (int j = j0; j < j1; ++j) nv += modality[j] != 0;
+        const int vbase = block_exclusive_scan(nv, scan_buf, &tot);
+        int neq = 0;
+        if (!none) {
+            int vr = vbase;
+            for (int j = j0; j < j1; ++j)
+                if (modality[j] != 0) {
+                    neq += (vr < p.N_v && keys[vr] == thr);
+                    ++vr;
+                }
+        }
+        const int ebase = block_exclusive_scan(neq, scan_buf, &tot);
+        // kept(j): text, or a vision key above T, or one of the first k_eq equal to T
+        auto scan_kept = [&](auto&& emit) {
+            int vr = vbase, er = ebase;
+            for (int j = j0; j < j1; ++j) {
+                bool keep = true;
+                if (modality[j] != 0) {
+                    keep = false;
+                    if (vr < p.N_v && !none) {
+                        const uint32_t key = keys[vr];
+                        if (key > thr) {
+                            keep = true;
+                        } else if (key == thr) {
+                            keep = er < k_eq;
+                            ++er;
+                        }
+                    }
+                    ++vr;
+                }
+                if (keep) emit(j);
+            }
+        };
+        int nkeep = 0;
+        scan_kept([&](int) { ++nkeep; });
+        const int kbase = block_exclusive_scan(nkeep, scan_buf, &tot);
+        off = s_off;
+        {
+            int r = kbase;
+            scan_kept([&](int j) {
+                if (r < len) {
+                    idx[off + r] = j;
+                    if (COMPACT) rows[r] = j;
+                }
+                ++r;
+            });
+        }
     }
     if (tid == 0 && tot != len) raise_status(status, TGVKV_STATUS_COUNT);
     if (!COMPACT) return;
