@@ -150,6 +150,8 @@ def stage_bytes(wl, ratio):
         "budget": 8 * wl.L,
         "select": scores + 4 * rows + 8 * (wl.L * wl.H_kv + 1),
         "compact": 4 * rows * wl.d * 2 + 4 * rows,
+        # the fused select + gather of tgvkv_evict (tgvkv_select_compact)
+        "tail": scores + 4 * rows * wl.d * 2 + 4 * rows + 8 * (wl.L * wl.H_kv + 1),
     }
 
 
@@ -258,6 +260,12 @@ def kernel_roof(wl, ratio, stage, launch_ms, peaks, peak_src="measured"):
     roof["bytes_per_launch"] = nbytes
     roof["flops_per_launch"] = flops
     return roof
+
+
+def _roof_brief(roof, launch_ms):
+    return {"launch_ms": launch_ms, "bound": roof["bound"], "achieved": roof["achieved"],
+            "unit": roof["unit"], "peak": roof["peak"], "frac": roof["frac"],
+            "bytes_per_launch": roof["bytes_per_launch"]}
 
 
 def mufu_of(wl, score_ms, clk_mhz):
@@ -542,8 +550,18 @@ def run_per_config(api, torch, dev, stream, barrier, seed, n_steps, inputs=None)
                     barrier()
                     return a.elapsed_time(b) / n_steps      # ms per call
 
+                def tail(i):
+                    # the evict's select + gather alone, on the last evict's
+                    # scores and budgets, K/V rotated as above
+                    x = sets[i % n_sets]
+                    api.tgvkv_select_compact(desc, out.scores, None, out.budgets, x["modality"],
+                                             x["k"], x["v"], out.offsets, out.idx, out.k_out,
+                                             out.v_out, ws, stream)
+
                 step_ms = timed(evict)
                 score_ms = timed(score)
+                evict(0)
+                tail_ms = timed(tail)
                 bits = api.tgvkv_status(ws, stream)
                 if bits != 0:
                     raise RuntimeError(f"device status bits 0x{bits:x} in {name} r={ratio}")
@@ -560,6 +578,8 @@ def run_per_config(api, torch, dev, stream, barrier, seed, n_steps, inputs=None)
                                      "share_of_step": score_ms / step_ms,
                                      "traffic": recorded_traffic("score", name)},
                     "score_mufu_frac": mufu_of(wl, score_ms, clk)["frac"],
+                    "tail_kernel": _roof_brief(kernel_roof(wl, ratio, "tail", tail_ms, peaks,
+                                                           peak_src), tail_ms),
                     "tail_ms": step_ms - score_ms, "rows_kept": rows, "steps": n_steps}
                 del out
             del sets, ws
@@ -650,9 +670,10 @@ def main():
     region_ms = float(region.item())
     us_per_layer = region_ms * 1e3 / (args.steps * wl.L * world)
 
-    # ---- per-stage breakdown (the four entry points with events between them)
-    stages = ["score", "budget", "select", "compact"]
-    sev = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
+    # ---- per-stage breakdown (the entry points with events between them; the
+    # fused select + gather follows the budget, as in the step)
+    stages = ["score", "budget", "tail", "select", "compact"]
+    sev = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(args.steps)]
     barrier()
     for s in range(args.steps):
         x = sets[s % n_sets]
@@ -663,12 +684,15 @@ def main():
         e[1].record(stream)
         api.tgvkv_budget(desc, out.tvb_stat, ratio, out.budgets, ws, stream)
         e[2].record(stream)
+        api.tgvkv_select_compact(desc, out.scores, None, out.budgets, x["modality"], x["k"], x["v"],
+                                 out.offsets, out.idx, out.k_out, out.v_out, ws, stream)
+        e[3].record(stream)
         api.tgvkv_select(desc, out.scores, out.budgets, x["modality"], out.offsets, out.idx, ws,
                          stream)
-        e[3].record(stream)
+        e[4].record(stream)
         api.tgvkv_compact(desc, x["k"], x["v"], out.offsets, out.idx, out.k_out, out.v_out, ws,
                           stream)
-        e[4].record(stream)
+        e[5].record(stream)
     barrier()
     stage_ms = {st: statistics.mean(sev[s][i].elapsed_time(sev[s][i + 1]) for s in range(args.steps))
                 for i, st in enumerate(stages)}
@@ -945,6 +969,10 @@ def main():
                          "launch_ms": stage_ms[dom],
                          "peak_source": roof["peak_source"], "frac_nominal": roof["frac_nominal"]},
             "score_mufu": mufu,
+            # the evict's fused select + gather timed alone after the budget
+            # (tgvkv_select_compact, the same kernel), against its own roof
+            "tail_kernel": _roof_brief(kernel_roof(wl, ratio, "tail", stage_ms["tail"], peaks,
+                                                   peak_src), stage_ms["tail"]),
             "stage_ms": stage_ms,
             "next_rows": next_rows,
             "decode": decode,

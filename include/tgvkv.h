@@ -232,6 +232,28 @@ int tgvkv_compact(const tgvkv_desc* desc, const uint16_t* k, const uint16_t* v,
                   uint16_t* k_out, uint16_t* v_out, int64_t capacity_rows,
                   void* workspace, void* stream);
 
+/* TPR retention and compaction in one pass (Eq. 10, then the gather): the
+ * tail of tgvkv_evict for scores and budgets the caller already holds.  The
+ * sets are those tgvkv_select_tpr makes (every option of the descriptor) and
+ * their rows those tgvkv_compact copies: offsets, idx, k_out and v_out as in
+ * those two calls.  scores, text_scores, budgets, modality: as in
+ * tgvkv_select_tpr; k, v: as in tgvkv_compact.
+ * capacity_rows: rows the caller allocated in each of idx, k_out and v_out
+ * (>= 0; tgvkv_retained_rows always suffices for budgets tgvkv_budget split
+ * from a ratio).  A set that would end past capacity_rows sets
+ * TGVKV_STATUS_INDEX and none of its indices or rows is written (offsets are
+ * written in full); a budget outside [0, cap] sets TGVKV_STATUS_BUDGET and is
+ * clamped.  One kernel for most shapes, or select then compact for sets too
+ * large for shared memory (tgvkv_select_compact_launches). */
+int tgvkv_select_compact(const tgvkv_desc* desc, const float* scores, const float* text_scores,
+                         const int32_t* budgets, const uint8_t* modality, const uint16_t* k,
+                         const uint16_t* v, int64_t* offsets, int32_t* idx, uint16_t* k_out,
+                         uint16_t* v_out, int64_t capacity_rows, void* workspace, void* stream);
+
+/* Kernel launches one tgvkv_select_compact call makes for desc (1 or 2; -1 on
+ * an invalid descriptor). */
+int tgvkv_select_compact_launches(const tgvkv_desc* desc);
+
 /* score -> budget -> select -> compact in one stream-ordered call with no host
  * synchronisation.  Arguments as in the four calls above.  With Eq. 7 weights
  * or the all-token basis it first runs tgvkv_text_scores into the workspace

@@ -48,6 +48,10 @@ SIGNATURES = {
                                  c_void_p, c_void_p, c_void_p]),
     "tgvkv_compact": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                               c_int64, c_void_p, c_void_p]),
+    "tgvkv_select_compact": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                     c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_int64,
+                                     c_void_p, c_void_p]),
+    "tgvkv_select_compact_launches": (c_int, [_P]),
     "tgvkv_evict": (c_int, [_P, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                             c_double, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                             c_void_p, c_void_p, c_void_p, c_void_p]),

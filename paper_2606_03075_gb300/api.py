@@ -212,6 +212,31 @@ def tgvkv_compact(desc, k, v, offsets, idx, k_out, v_out, ws, stream=None):
         _stream(stream)), "tgvkv_compact")
 
 
+def tgvkv_select_compact(desc, scores, text_scores, budgets, modality, k, v, offsets, idx,
+                         k_out, v_out, ws, stream=None):
+    LH = desc.L * desc.H_kv
+    n = LH * desc.N * desc.d
+    # rows every output holds: k_out, v_out and idx alike
+    capacity = min(k_out.numel() // desc.d, v_out.numel() // desc.d, idx.numel())
+    _check(_lib.load().tgvkv_select_compact(
+        ctypes.byref(desc),
+        _ptr(scores, (torch.float32,), LH * desc.N_v, "scores"),
+        _ptr(text_scores, (torch.float32,), LH * (desc.N - desc.N_v), "text_scores"),
+        _ptr(budgets, (torch.int32,), budget_units(desc), "budgets"),
+        _ptr(modality, (torch.uint8,), desc.N, "modality"),
+        _ptr(k, _BF16_LIKE, n, "k"), _ptr(v, _BF16_LIKE, n, "v"),
+        _ptr(offsets, (torch.int64,), LH + 1, "offsets"),
+        _ptr(idx, (torch.int32,), 0, "idx"),
+        _ptr(k_out, _BF16_LIKE, 0, "k_out"), _ptr(v_out, _BF16_LIKE, 0, "v_out"),
+        capacity,
+        _ptr(ws, (torch.uint8,), tgvkv_workspace_size(desc), "workspace"),
+        _stream(stream)), "tgvkv_select_compact")
+
+
+def tgvkv_select_compact_launches(desc: Desc) -> int:
+    return int(_lib.load().tgvkv_select_compact_launches(ctypes.byref(desc)))
+
+
 @dataclass
 class EvictOutputs:
     scores: torch.Tensor     # fp32 [L, H_kv, N_v]

@@ -452,6 +452,41 @@ int tgvkv_compact(const tgvkv_desc* desc, const uint16_t* k, const uint16_t* v,
     return e == cudaSuccess ? ok() : cuda_fail(e, "compact launch");
 }
 
+int tgvkv_select_compact(const tgvkv_desc* desc, const float* scores, const float* text_scores,
+                         const int32_t* budgets, const uint8_t* modality, const uint16_t* k,
+                         const uint16_t* v, int64_t* offsets, int32_t* idx, uint16_t* k_out,
+                         uint16_t* v_out, int64_t capacity_rows, void* workspace, void* stream) {
+    Problem p{};
+    int rc = make_problem(desc, &p);
+    if (rc) return rc;
+    if (capacity_rows < 0) return fail(TGVKV_ERR_INVALID_ARG, "capacity_rows %lld < 0",
+                                       (long long)capacity_rows);
+    if (p.N_v > 0) REQUIRE_PTR(scores, "scores", false);
+    if (p.basis == TGVKV_BASIS_ALL && p.N_t > 0) REQUIRE_PTR(text_scores, "text_scores", false);
+    REQUIRE_PTR(budgets, "budgets", false);
+    REQUIRE_PTR(modality, "modality", false);
+    REQUIRE_PTR(k, "k", true);
+    REQUIRE_PTR(v, "v", true);
+    REQUIRE_PTR(offsets, "offsets", false);
+    REQUIRE_PTR(idx, "idx", false);
+    REQUIRE_PTR(k_out, "k_out", true);
+    REQUIRE_PTR(v_out, "v_out", true);
+    REQUIRE_PTR(workspace, "workspace", true);
+    const WsLayout lay = layout_of(p);
+    // every set holds at most N rows: no more can be asked of the kernels
+    const long long cap = std::min((long long)capacity_rows, (long long)p.L * p.H_kv * p.N);
+    cudaError_t e = launch_select_compact(p, scores, text_scores, budgets, modality, offsets, idx,
+                                          k, v, k_out, v_out, cap, status_of(workspace, lay),
+                                          static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ok() : cuda_fail(e, "select/compact launch");
+}
+
+int tgvkv_select_compact_launches(const tgvkv_desc* desc) {
+    Problem p{};
+    if (make_problem(desc, &p)) return -1;
+    return select_compact_launches(p);
+}
+
 int tgvkv_evict(const tgvkv_desc* desc, const uint16_t* q_text, const uint16_t* k,
                 const uint16_t* v, const uint8_t* modality, const int32_t* text_pos,
                 const float* w, double ratio, float* scores, float* tvb_stat, int32_t* budgets,

@@ -17,7 +17,7 @@ __global__ void __launch_bounds__(kThreads)
 compact_kernel(Problem p, const uint4* __restrict__ k, const uint4* __restrict__ v,
                const int64_t* __restrict__ offsets, const int32_t* __restrict__ idx,
                uint4* __restrict__ k_out, uint4* __restrict__ v_out, long long capacity,
-               uint32_t* __restrict__ status) {
+               int whole_sets, uint32_t* __restrict__ status) {
     constexpr int RPI = 32 / VPR;                 // rows per warp per iteration
     constexpr int ROWS_PER_WARP = RPI * kIter;
     constexpr int ROWS_PER_CTA = ROWS_PER_WARP * (kThreads / 32);
@@ -54,6 +54,9 @@ compact_kernel(Problem p, const uint4* __restrict__ k, const uint4* __restrict__
         ok[it] = r < total;
         if (ok[it]) {
             while (offsets[lg + 1] <= r) ++lg;
+            if (whole_sets && offsets[lg + 1] > capacity) ok[it] = false;   // its set does not fit
+        }
+        if (ok[it]) {
             const int src = idx[r];
             if (src < 0 || src >= p.N) {
                 raise_status(status, TGVKV_STATUS_INDEX);
@@ -77,14 +80,15 @@ compact_kernel(Problem p, const uint4* __restrict__ k, const uint4* __restrict__
 template <int VPR>
 cudaError_t launch_compact_t(const Problem& p, const uint16_t* k, const uint16_t* v,
                              const int64_t* offsets, const int32_t* idx, uint16_t* k_out,
-                             uint16_t* v_out, long long capacity_rows, uint32_t* status,
-                             cudaStream_t stream) {
+                             uint16_t* v_out, long long capacity_rows, bool whole_sets,
+                             uint32_t* status, cudaStream_t stream) {
     constexpr int ROWS_PER_CTA = (32 / VPR) * kIter * (kThreads / 32);
     const long long blocks = (capacity_rows + ROWS_PER_CTA - 1) / ROWS_PER_CTA;
     if (blocks == 0) return cudaSuccess;
     compact_kernel<VPR><<<(unsigned)blocks, kThreads, 0, stream>>>(
         p, reinterpret_cast<const uint4*>(k), reinterpret_cast<const uint4*>(v), offsets, idx,
-        reinterpret_cast<uint4*>(k_out), reinterpret_cast<uint4*>(v_out), capacity_rows, status);
+        reinterpret_cast<uint4*>(k_out), reinterpret_cast<uint4*>(v_out), capacity_rows,
+        whole_sets ? 1 : 0, status);
     return cudaGetLastError();
 }
 
@@ -93,10 +97,12 @@ cudaError_t launch_compact_t(const Problem& p, const uint16_t* k, const uint16_t
 cudaError_t launch_compact(const Problem& p, const uint16_t* k, const uint16_t* v,
                            const int64_t* offsets, const int32_t* idx, uint16_t* k_out,
                            uint16_t* v_out, long long capacity_rows, uint32_t* status,
-                           cudaStream_t stream) {
+                           cudaStream_t stream, bool whole_sets) {
     if (p.d == 64)
-        return launch_compact_t<8>(p, k, v, offsets, idx, k_out, v_out, capacity_rows, status, stream);
-    return launch_compact_t<16>(p, k, v, offsets, idx, k_out, v_out, capacity_rows, status, stream);
+        return launch_compact_t<8>(p, k, v, offsets, idx, k_out, v_out, capacity_rows, whole_sets,
+                                   status, stream);
+    return launch_compact_t<16>(p, k, v, offsets, idx, k_out, v_out, capacity_rows, whole_sets,
+                                status, stream);
 }
 
 }  // namespace tgvkv

@@ -93,9 +93,11 @@ int device_sm_count();
 // arrives at; the wait runs out and sets TGVKV_STATUS_TIMEOUT (selftest.cu).
 cudaError_t launch_wait_timeout(uint32_t* status, cudaStream_t stream);
 
+// Compaction (compact.cu).  Rows from capacity_rows on are never written;
+// with whole_sets, neither is any row of a set that ends past capacity_rows.
 cudaError_t launch_compact(const Problem& p, const uint16_t* k, const uint16_t* v,
                            const int64_t* offsets, const int32_t* idx, uint16_t* k_out,
                            uint16_t* v_out, long long capacity_rows, uint32_t* status,
-                           cudaStream_t stream);
+                           cudaStream_t stream, bool whole_sets = false);
 
 }  // namespace tgvkv

@@ -138,7 +138,7 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
                   const uint8_t* __restrict__ modality_g, int64_t* __restrict__ offsets,
                   int32_t* __restrict__ idx, const uint4* __restrict__ k,
                   const uint4* __restrict__ v, uint4* __restrict__ k_out,
-                  uint4* __restrict__ v_out, uint32_t* __restrict__ status) {
+                  uint4* __restrict__ v_out, long long capacity, uint32_t* __restrict__ status) {
     extern __shared__ __align__(16) unsigned char dyn_raw[];
     uint32_t* keys = reinterpret_cast<uint32_t*>(dyn_raw);  // [N_v]
     int* rows = reinterpret_cast<int*>(keys + p.N_v);       // [N_t + b] (gather form)
@@ -149,7 +149,6 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
     __shared__ uint32_t s_prefix;
     __shared__ int s_kk;
     __shared__ int s_ties;
-    __shared__ long long s_off;
 
     // fused form: CTA 2h selects head h and gathers its interior rows, CTA
     // 2h + 1 copies its edge rows
@@ -181,12 +180,21 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
         if (lane == 0) off_part[warp] = part;
     }
     __syncthreads();
+    // the set's first row, the same in every thread (recomputed where needed
+    // rather than held in registers across the selection)
+    auto set_offset = [&]() {
+        long long o = (long long)g * len;
+        for (int w = 0; w < kThreads / 32; ++w) o += off_part[w];
+        return o;
+    };
+    // a set that would end past the caller's rows writes none of its rows or indices
+    const bool fits = set_offset() + len <= capacity;
     int vlo = 0, vhi = 0;   // edge rows: positions [0, vlo) and [vhi, N)
     if (COMPACT) vision_span_block(modality, p.N, &vlo, &vhi, span_red);
     if (vhi < vlo) vhi = vlo;   // no vision key: every row is a leading edge row
     if (edge_cta) {
-        long long off = (long long)g * len;
-        for (int w = 0; w < kThreads / 32; ++w) off += off_part[w];
+        if (!fits) return;
+        const long long off = set_offset();
         const size_t head = (size_t)lg * p.N;
         const int tail = p.N - vhi;
         if (vlo <= len) copy_rows<VPR>(k, v, k_out, v_out, head, 0, off, vlo, tid, kThreads);
@@ -194,16 +202,16 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
             copy_rows<VPR>(k, v, k_out, v_out, head, vhi, off + len - tail, tail, tid, kThreads);
         return;
     }
+    if (tid == 0) {
+        const long long off = set_offset();
+        offsets[lg] = off;
+        if (lg == p.L * p.H_kv - 1) offsets[lg + 1] = off + len;
+        if (!fits) raise_status(status, TGVKV_STATUS_INDEX);
+    }
+    if (!fits) return;
     const float* sc = scores + (size_t)lg * p.N_v;
     for (int i = tid; i < p.N_v; i += kThreads) keys[i] = float_order_key(__ldg(sc + i));
     __syncthreads();
-    if (tid == 0) {
-        long long off = (long long)g * len;
-        for (int w = 0; w < kThreads / 32; ++w) off += off_part[w];
-        s_off = off;
-        offsets[lg] = off;
-        if (lg == p.L * p.H_kv - 1) offsets[lg + 1] = off + len;
-    }
 
     // ---- radix select of the b-th largest key
     uint32_t prefix = 0;
@@ -257,7 +265,7 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
     const uint32_t thr = prefix;
     const int k_eq = none ? 0 : kk;
     int tot;
-    long long off;   // read from s_off after a block barrier (with b = 0 no round runs)
+    const long long off = set_offset();
 
     if (none || s_ties == k_eq) {
         // ---- every key equal to T is kept (no ties to break): a vision key
@@ -274,7 +282,6 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
             nvw += __popc(__ballot_sync(~0u, j < w1 && modality[j] != 0));
         }
         const int vbase = __shfl_sync(~0u, block_exclusive_scan(lane == 0 ? nvw : 0, scan_buf, &tot), 0);
-        off = s_off;
         auto walk = [&](auto&& emit) {
             int vr = vbase, kr = 0;
             for (int c0 = w0; c0 < w1; c0 += 32) {
@@ -342,7 +349,6 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
         int nkeep = 0;
         scan_kept([&](int) { ++nkeep; });
         const int kbase = block_exclusive_scan(nkeep, scan_buf, &tot);
-        off = s_off;
         {
             int r = kbase;
             scan_kept([&](int j) {
@@ -406,7 +412,7 @@ tpr_select_warp_kernel(Problem p, const float* __restrict__ scores,
                        int64_t* __restrict__ offsets, int32_t* __restrict__ idx,
                        const uint4* __restrict__ k, const uint4* __restrict__ v,
                        uint4* __restrict__ k_out, uint4* __restrict__ v_out,
-                       uint32_t* __restrict__ status) {
+                       long long capacity, uint32_t* __restrict__ status) {
     extern __shared__ __align__(16) unsigned char dyn_raw[];
     const int wid = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nw = blockDim.x >> 5;
@@ -447,8 +453,10 @@ tpr_select_warp_kernel(Problem p, const float* __restrict__ scores,
     off += (long long)g * len;
     const int tail = p.N - vhi;
     const bool edges_ok = vlo <= len && tail <= len - vlo;
+    // a set that would end past the caller's rows writes none of its rows or indices
+    const bool fits = off + len <= capacity;
     if (edge_cta) {
-        if (edges_ok) {
+        if (edges_ok && fits) {
             const size_t head = (size_t)lg * p.N;
             copy_rows<VPR>(k, v, k_out, v_out, head, 0, off, vlo, lane, 32);
             copy_rows<VPR>(k, v, k_out, v_out, head, vhi, off + len - tail, tail, lane, 32);
@@ -458,7 +466,9 @@ tpr_select_warp_kernel(Problem p, const float* __restrict__ scores,
     if (lane == 0) {
         offsets[lg] = off;
         if (lg == p.L * p.H_kv - 1) offsets[lg + 1] = off + len;
+        if (!fits) raise_status(status, TGVKV_STATUS_INDEX);
     }
+    if (!fits) return;
     const float* sc = scores + (size_t)lg * p.N_v;
     for (int i = lane; i < p.N_v; i += 32) keys[i] = float_order_key(__ldg(sc + i));
     __syncwarp();
@@ -622,7 +632,7 @@ tpr_select_general_kernel(Problem p, const float* __restrict__ scores,
                           int64_t* __restrict__ offsets, int32_t* __restrict__ idx,
                           const uint4* __restrict__ k, const uint4* __restrict__ v,
                           uint4* __restrict__ k_out, uint4* __restrict__ v_out,
-                          uint32_t* __restrict__ status) {
+                          long long capacity, uint32_t* __restrict__ status) {
     extern __shared__ __align__(16) unsigned char dyn_raw[];
     const size_t keyset = (size_t)(p.N_v > p.N_t ? p.N_v : p.N_t);
     uint32_t* keys = reinterpret_cast<uint32_t*>(dyn_raw);          // [candidates]
@@ -706,6 +716,11 @@ tpr_select_general_kernel(Problem p, const float* __restrict__ scores,
     const float* sc = c.vision ? scores + (size_t)lg * p.N_v : text_scores + (size_t)lg * p.N_t;
     for (int i = tid; i < n_cand; i += kThreads) keys[i] = float_order_key(__ldg(sc + i));
     __syncthreads();
+    // a set that would end past the caller's rows writes none of its rows or indices
+    if (s_off + len > capacity) {
+        if (tid == 0) raise_status(status, TGVKV_STATUS_INDEX);
+        return;
+    }
 
     // ---- candidate ranks of each thread's contiguous position range; sinks get key 0
     const int per = (p.N + kThreads - 1) / kThreads;
@@ -857,7 +872,8 @@ template <bool COMPACT, int VPR>
 cudaError_t launch_sel_general(const Problem& p, const float* scores, const float* text_scores,
                                const int32_t* budgets, const uint8_t* modality, int64_t* offsets,
                                int32_t* idx, const uint16_t* k, const uint16_t* v, uint16_t* k_out,
-                               uint16_t* v_out, uint32_t* status, cudaStream_t stream) {
+                               uint16_t* v_out, long long capacity, uint32_t* status,
+                               cudaStream_t stream) {
     auto kern = tpr_select_general_kernel<COMPACT, VPR>;
     const size_t smem = select_general_smem(p, COMPACT);
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -865,7 +881,7 @@ cudaError_t launch_sel_general(const Problem& p, const float* scores, const floa
     kern<<<p.L * p.H_kv, kThreads, smem, stream>>>(
         p, scores, text_scores, budgets, modality, offsets, idx, reinterpret_cast<const uint4*>(k),
         reinterpret_cast<const uint4*>(v), reinterpret_cast<uint4*>(k_out),
-        reinterpret_cast<uint4*>(v_out), status);
+        reinterpret_cast<uint4*>(v_out), capacity, status);
     return cudaGetLastError();
 }
 
@@ -889,7 +905,7 @@ template <int VPR>
 cudaError_t launch_sel_warp(const Problem& p, int nw, const float* scores, const int32_t* budgets,
                             const uint8_t* modality, int64_t* offsets, int32_t* idx,
                             const uint16_t* k, const uint16_t* v, uint16_t* k_out, uint16_t* v_out,
-                            uint32_t* status, cudaStream_t stream) {
+                            long long capacity, uint32_t* status, cudaStream_t stream) {
     auto kern = tpr_select_warp_kernel<VPR>;
     const size_t smem = (((size_t)p.N + 15) & ~size_t(15)) + sizeof(uint32_t) * warp_select_words(p) * nw;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -898,7 +914,7 @@ cudaError_t launch_sel_warp(const Problem& p, int nw, const float* scores, const
     kern<<<2 * ((heads + nw - 1) / nw), nw * 32, smem, stream>>>(
         p, scores, budgets, modality, offsets, idx, reinterpret_cast<const uint4*>(k),
         reinterpret_cast<const uint4*>(v), reinterpret_cast<uint4*>(k_out),
-        reinterpret_cast<uint4*>(v_out), status);
+        reinterpret_cast<uint4*>(v_out), capacity, status);
     return cudaGetLastError();
 }
 
@@ -906,7 +922,7 @@ template <bool COMPACT, int VPR>
 cudaError_t launch_sel(const Problem& p, const float* scores, const int32_t* budgets,
                        const uint8_t* modality, int64_t* offsets, int32_t* idx,
                        const uint16_t* k, const uint16_t* v, uint16_t* k_out, uint16_t* v_out,
-                       uint32_t* status, cudaStream_t stream) {
+                       long long capacity, uint32_t* status, cudaStream_t stream) {
     auto kern = tpr_select_kernel<COMPACT, VPR>;
     const size_t smem = select_smem(p, COMPACT);
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -915,8 +931,25 @@ cudaError_t launch_sel(const Problem& p, const float* scores, const int32_t* bud
         p, scores, budgets, modality, offsets, idx,
         reinterpret_cast<const uint4*>(k),
         reinterpret_cast<const uint4*>(v), reinterpret_cast<uint4*>(k_out),
-        reinterpret_cast<uint4*>(v_out), status);
+        reinterpret_cast<uint4*>(v_out), capacity, status);
     return cudaGetLastError();
+}
+
+// The select-only form writes no rows; its index capacity is the caller's
+// (tgvkv_retained_rows for sets of a split the budget call made).
+constexpr long long kNoCapacity = 0x7FFFFFFFFFFFFFFFLL;
+
+// Select only; a set that would end past `capacity` indices writes none.
+cudaError_t launch_select_cap(const Problem& p, const float* scores, const float* text_scores,
+                              const int32_t* budgets, const uint8_t* modality, int64_t* offsets,
+                              int32_t* idx, long long capacity, uint32_t* status,
+                              cudaStream_t stream) {
+    if (general_select(p))
+        return launch_sel_general<false, 16>(p, scores, text_scores, budgets, modality, offsets,
+                                             idx, nullptr, nullptr, nullptr, nullptr, capacity,
+                                             status, stream);
+    return launch_sel<false, 16>(p, scores, budgets, modality, offsets, idx, nullptr, nullptr, nullptr,
+                                 nullptr, capacity, status, stream);
 }
 
 }  // namespace
@@ -924,12 +957,8 @@ cudaError_t launch_sel(const Problem& p, const float* scores, const int32_t* bud
 cudaError_t launch_select(const Problem& p, const float* scores, const float* text_scores,
                           const int32_t* budgets, const uint8_t* modality, int64_t* offsets,
                           int32_t* idx, uint32_t* status, cudaStream_t stream) {
-    if (general_select(p))
-        return launch_sel_general<false, 16>(p, scores, text_scores, budgets, modality, offsets,
-                                             idx, nullptr, nullptr, nullptr, nullptr, status,
-                                             stream);
-    return launch_sel<false, 16>(p, scores, budgets, modality, offsets, idx, nullptr, nullptr, nullptr,
-                                 nullptr, status, stream);
+    return launch_select_cap(p, scores, text_scores, budgets, modality, offsets, idx, kNoCapacity,
+                             status, stream);
 }
 
 int select_compact_launches(const Problem& p) {
@@ -944,36 +973,38 @@ cudaError_t launch_select_compact(const Problem& p, const float* scores, const f
                                   long long capacity_rows, uint32_t* status, cudaStream_t stream) {
     if (general_select(p)) {
         if (select_general_smem(p, true) > kFusedSmemLimit) {
-            cudaError_t e = launch_select(p, scores, text_scores, budgets, modality, offsets, idx,
-                                          status, stream);
+            cudaError_t e = launch_select_cap(p, scores, text_scores, budgets, modality, offsets,
+                                              idx, capacity_rows, status, stream);
             if (e != cudaSuccess) return e;
             return launch_compact(p, k, v, offsets, idx, k_out, v_out, capacity_rows, status,
-                                  stream);
+                                  stream, /*whole_sets=*/true);
         }
         if (p.d == 64)
             return launch_sel_general<true, 8>(p, scores, text_scores, budgets, modality, offsets,
-                                               idx, k, v, k_out, v_out, status, stream);
+                                               idx, k, v, k_out, v_out, capacity_rows, status,
+                                               stream);
         return launch_sel_general<true, 16>(p, scores, text_scores, budgets, modality, offsets, idx,
-                                            k, v, k_out, v_out, status, stream);
+                                            k, v, k_out, v_out, capacity_rows, status, stream);
     }
     if (const int nw = warp_select_warps(p)) {
         if (p.d == 64)
             return launch_sel_warp<8>(p, nw, scores, budgets, modality, offsets, idx, k, v, k_out,
-                                      v_out, status, stream);
+                                      v_out, capacity_rows, status, stream);
         return launch_sel_warp<16>(p, nw, scores, budgets, modality, offsets, idx, k, v, k_out,
-                                   v_out, status, stream);
+                                   v_out, capacity_rows, status, stream);
     }
     if (select_smem(p, true) > kFusedSmemLimit) {
-        cudaError_t e = launch_select(p, scores, nullptr, budgets, modality, offsets, idx, status,
-                                      stream);
+        cudaError_t e = launch_select_cap(p, scores, nullptr, budgets, modality, offsets, idx,
+                                          capacity_rows, status, stream);
         if (e != cudaSuccess) return e;
-        return launch_compact(p, k, v, offsets, idx, k_out, v_out, capacity_rows, status, stream);
+        return launch_compact(p, k, v, offsets, idx, k_out, v_out, capacity_rows, status, stream,
+                              /*whole_sets=*/true);
     }
     if (p.d == 64)
         return launch_sel<true, 8>(p, scores, budgets, modality, offsets, idx, k, v, k_out, v_out,
-                                   status, stream);
+                                   capacity_rows, status, stream);
     return launch_sel<true, 16>(p, scores, budgets, modality, offsets, idx, k, v, k_out, v_out,
-                                status, stream);
+                                capacity_rows, status, stream);
 }
 
 }  // namespace tgvkv

@@ -144,6 +144,33 @@ def test_evict_launch_count_with_text_pass(lib):
         assert lib.tgvkv_evict_launches(ref(_desc(**base, keep_first=4, keep_last=1))) == 2
 
 
+def test_select_compact_launch_count_and_validation(lib):
+    """tgvkv_select_compact: the one fused kernel wherever tgvkv_evict uses it
+    (select then compact for sets too large for shared memory), and host-side
+    rejection of a negative capacity and of missing or misaligned buffers."""
+    ref = ctypes.byref
+    for wl in synth.WORKLOADS.values():
+        d = _desc(L=wl.L, H_q=wl.H_q, H_kv=wl.H_kv, d=wl.d, N=wl.N, N_v=wl.N_v, n_win=wl.n_win,
+                  w_layer_stride=wl.n_win)
+        assert lib.tgvkv_select_compact_launches(ref(d)) == 1, wl.name
+        assert lib.tgvkv_select_compact_launches(ref(_desc(**{**dict(
+            L=wl.L, H_q=wl.H_q, H_kv=wl.H_kv, d=wl.d, N=wl.N, N_v=wl.N_v, n_win=wl.n_win,
+            w_layer_stride=wl.n_win), "keep_first": 4, "keep_last": 1}))) == 1, wl.name
+    assert lib.tgvkv_select_compact_launches(ref(_desc(N=32000, N_v=31000))) == 2
+    assert lib.tgvkv_select_compact_launches(ref(_desc(d=32))) == -1
+    assert lib.tgvkv_select_compact_launches(None) == -1
+    P = ctypes.c_void_p
+    fake, odd = P(0x1000), P(0x1008)   # never dereferenced: each call fails validation
+
+    def call(cap=16, k=fake, k_out=fake, ws=fake, scores=fake):
+        return lib.tgvkv_select_compact(ref(_desc()), scores, None, fake, fake, k, fake, fake,
+                                        fake, k_out, fake, cap, ws, None)
+
+    assert call(cap=-1) == 1
+    assert call(k=odd) == 1 and call(k_out=odd) == 1
+    assert call(ws=None) == 1 and call(scores=None) == 1
+
+
 def test_decode_launch_count(lib):
     """Two decode kernels for every shape: the row streams, then the merge of
     the sets they split (launched as a programmatic dependent)."""
