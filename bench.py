@@ -499,10 +499,12 @@ PER_CONFIG = [("tiny", 0.25), ("llava15", 0.05), ("llava15", 0.20), ("next", 0.0
 
 
 def run_per_config(api, torch, dev, stream, barrier, seed, n_steps, inputs=None):
-    """The fused step (tgvkv_evict) and its score kernel alone (tgvkv_score) on
-    every workload and budget: n_steps timed calls each after 3 warm-up calls,
-    inputs rotated past L2.  Returns {"<name> r=<ratio>": {...}} and the clocks
-    seen over the whole block."""
+    """The fused step (tgvkv_evict), its score kernel alone (tgvkv_score), its
+    select + gather alone (tgvkv_select_compact) and one decode step over the
+    compacted cache it made (tgvkv_decode) on every workload and budget:
+    n_steps timed calls each after 3 warm-up calls, inputs rotated past L2.
+    Returns {"<name> r=<ratio>": {...}} and the clocks seen over the whole
+    block."""
     peaks, peak_src = measured_peaks()
     hbm_peak = float(peaks["hbm_gbs"])
     res = {}
@@ -562,6 +564,26 @@ def run_per_config(api, torch, dev, stream, barrier, seed, n_steps, inputs=None)
                 score_ms = timed(score)
                 evict(0)
                 tail_ms = timed(tail)
+
+                # one decode step over the compacted cache this step made (the
+                # consumer), copies of the cache rotated past L2
+                n_rows = int(out.offsets[-1].item())
+                comp_bytes = 2 * n_rows * wl.d * 2
+                n_cp = max(2, math.ceil(2 * L2_BYTES / max(comp_bytes, 1)) + 1)
+                comp = [(out.k_out[:n_rows].clone(), out.v_out[:n_rows].clone())
+                        for _ in range(n_cp)]
+                offs = out.offsets.clone()
+                qdec = torch.from_numpy(synth.to_bf16_bits(
+                    np.random.default_rng(seed + 11).standard_normal((wl.L, wl.H_q, wl.d))
+                    .astype(np.float32))).to(dev).view(torch.bfloat16)
+                odec = torch.empty((wl.L, wl.H_q, wl.d), dtype=torch.float32, device=dev)
+
+                def decode(i):
+                    kk, vv = comp[i % n_cp]
+                    api.tgvkv_decode(desc, qdec, kk, vv, offs, odec, ws, stream)
+
+                dec_ms = timed(decode)
+                del comp
                 bits = api.tgvkv_status(ws, stream)
                 if bits != 0:
                     raise RuntimeError(f"device status bits 0x{bits:x} in {name} r={ratio}")
@@ -580,7 +602,11 @@ def run_per_config(api, torch, dev, stream, barrier, seed, n_steps, inputs=None)
                     "score_mufu_frac": mufu_of(wl, score_ms, clk)["frac"],
                     "tail_kernel": _roof_brief(kernel_roof(wl, ratio, "tail", tail_ms, peaks,
                                                            peak_src), tail_ms),
-                    "tail_ms": step_ms - score_ms, "rows_kept": rows, "steps": n_steps}
+                    "tail_ms": step_ms - score_ms, "rows_kept": rows, "steps": n_steps,
+                    "decode": {"us_per_token": dec_ms * 1e3,
+                               "gbs": comp_bytes / (dec_ms * 1e-3) / 1e9,
+                               "frac": comp_bytes / (dec_ms * 1e-3) / 1e9 / hbm_peak,
+                               "rows": n_rows}}
                 del out
             del sets, ws
             torch.cuda.empty_cache()
