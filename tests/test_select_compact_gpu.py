@@ -163,3 +163,29 @@ def test_select_compact_matches_evict_tail(api):
     assert torch.equal(idx[:n], out.idx[:n])
     assert torch.equal(ko[:n].view(torch.int16), out.k_out[:n].view(torch.int16))
     assert torch.equal(vo[:n].view(torch.int16), out.v_out[:n].view(torch.int16))
+
+
+@pytest.mark.parametrize("name", ["cta", "cta_d64", "warp"])
+@pytest.mark.parametrize("extra", [0, -1, 1])
+def test_select_ties_at_the_threshold(api, name, extra):
+    """Scores of three values in known counts.  With b = #(score >= 2) every
+    key equal to the threshold is kept (the kernels' no-tie emission); with
+    b - 1 or b + 1 the keys equal to the threshold (2, or 1) must be broken by
+    position (the tie-breaking emission).  Against the oracle's Eq. 10 sets."""
+    x = _inputs(name, 13, False)
+    rng = np.random.default_rng(14)
+    L, H, N_v = x["L"], x["H"], x["N_v"]
+    sc = rng.choice(np.array([1.0, 2.0, 3.0], np.float32), size=(L, H, N_v), p=[0.6, 0.3, 0.1])
+    sc[:, :, 0] = 2.0                          # at least one key at the threshold in every head
+    x["sc"] = sc.astype(np.float32)
+    # one budget per layer, from the head with the fewest keys >= 2 (every head can fill it)
+    ge2 = (sc >= 2.0).sum(axis=2).min(axis=1)
+    x["budgets"] = np.clip(ge2 + extra, 0, N_v).astype(np.int32)
+    r_off, r_idx, r_ko, r_vo = _oracle(x, "vision", (0, 0))
+    total = int(r_off[-1])
+    _, status, off, idx, ko, vo = _run(api, x, "vision", (0, 0), capacity=total)
+    assert status == 0
+    np.testing.assert_array_equal(off, r_off)
+    np.testing.assert_array_equal(idx[:total], r_idx)
+    np.testing.assert_array_equal(ko[:total], r_ko)
+    np.testing.assert_array_equal(vo[:total], r_vo)
