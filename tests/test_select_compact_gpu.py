@@ -189,3 +189,34 @@ def test_select_ties_at_the_threshold(api, name, extra):
     np.testing.assert_array_equal(idx[:total], r_idx)
     np.testing.assert_array_equal(ko[:total], r_ko)
     np.testing.assert_array_equal(vo[:total], r_vo)
+
+
+@pytest.mark.parametrize("name", ["cta", "warp", "split"])
+def test_select_compact_head_budgets(api, name):
+    """One budget per (layer, KV head) (the head-adaptive option): the sets of
+    Eq. 10 with each head's own b, against the oracle."""
+    x = _inputs(name, 15, False)
+    rng = np.random.default_rng(16)
+    L, H, N_v = x["L"], x["H"], x["N_v"]
+    hb = rng.integers(0, N_v + 1, (L, H)).astype(np.int32)
+    hb[0, 0] = 0
+    hb[-1, -1] = N_v
+    off_r, idx_r = oracle.tpr_select_general(x["sc"].astype(np.float64), x["ts"].astype(np.float64),
+                                             hb, x["modality"], 0, 0, vision_basis=True)
+    ko_r, vo_r = oracle.compact(x["k"], x["v"], off_r, idx_r)
+    total = int(off_r[-1])
+    desc = api.make_desc(L, H, H, x["d"], x["N"], N_v, 1, head_budgets=True)
+    ws = api.new_workspace(desc)
+    dev = lambda a: torch.from_numpy(np.ascontiguousarray(a)).cuda()
+    off = torch.empty(L * H + 1, dtype=torch.int64, device="cuda")
+    idx = torch.empty(total, dtype=torch.int32, device="cuda")
+    ko = torch.empty((total, x["d"]), dtype=torch.int16, device="cuda")
+    vo = torch.empty_like(ko)
+    api.tgvkv_select_compact(desc, dev(x["sc"]), None, dev(hb.reshape(-1)), dev(x["modality"]),
+                             dev(x["k"]).view(torch.bfloat16), dev(x["v"]).view(torch.bfloat16),
+                             off, idx, ko.view(torch.bfloat16), vo.view(torch.bfloat16), ws)
+    assert api.tgvkv_status(ws) == 0
+    np.testing.assert_array_equal(off.cpu().numpy(), off_r)
+    np.testing.assert_array_equal(idx.cpu().numpy(), idx_r)
+    np.testing.assert_array_equal(ko.cpu().numpy(), ko_r)
+    np.testing.assert_array_equal(vo.cpu().numpy(), vo_r)
