@@ -110,4 +110,66 @@ __device__ __forceinline__ void tvb_budget_block(const float* stat, int L, long 
         for (int l = tid; l < L; l += nt) budgets[l] = b.result[l];
 }
 
+// tvb_budget_block for at most 32 units, by one warp (lane l = unit l, every
+// lane of the warp calling): the same double operations in the same order --
+// the denominator summed over the active units in unit order, the quotient
+// rounded multiply then rounded divide, the fractional part's bit pattern
+// ranked (fraction desc, unit asc) -- so the same integers, with warp
+// shuffles in place of the block's shared scratch and barriers.  stat: the
+// statistic of unit `lane` (ignored when uniform).
+__device__ __forceinline__ void tvb_budget_warp(float stat, int L, long long total, int cap,
+                                                int32_t* budgets, uint32_t* status, bool uniform,
+                                                int lane) {
+    const bool has = lane < L;
+    const double st = (has && !uniform) ? (double)stat : 0.0;
+    bool active = has;
+    int result = 0;
+    long long remaining = total;
+    int n_active = L;
+    for (int round = 0; round <= L; ++round) {
+        const uint32_t act = __ballot_sync(~0u, active);
+        double den = 0.0;
+        for (int m = 0; m < L; ++m) {
+            const double sm = __shfl_sync(~0u, st, m);
+            if ((act >> m) & 1u) den = __dadd_rn(den, sm);
+        }
+        const double rem = (double)remaining;
+        long long base = 0;
+        unsigned long long frac = 0;
+        if (active) {
+            const double qv = den > 0.0 ? __ddiv_rn(__dmul_rn(rem, st), den)
+                                        : __ddiv_rn(rem, (double)n_active);
+            const double fl = floor(qv);
+            base = (long long)fl;
+            frac = (unsigned long long)__double_as_longlong(__dsub_rn(qv, fl));
+        }
+        long long floors = base;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) floors += __shfl_xor_sync(~0u, floors, o);
+        const long long leftover = remaining - floors;
+        long long rank = 0;
+        for (int m = 0; m < L; ++m) {
+            const unsigned long long fm = __shfl_sync(~0u, frac, m);
+            if (active && ((act >> m) & 1u) && m != lane && (fm > frac || (fm == frac && m < lane)))
+                ++rank;
+        }
+        const long long v = base + (rank < leftover ? 1 : 0);
+        const uint32_t over = __ballot_sync(~0u, active && v > cap);
+        if (over == 0u) {
+            if (active) result = (int)v;
+            break;
+        }
+        if ((over >> lane) & 1u) {
+            active = false;
+            result = cap;
+        }
+        const int n_over = __popc(over);
+        remaining -= (long long)cap * n_over;
+        n_active -= n_over;
+        if (n_active == 0 && remaining != 0 && lane == 0) raise_status(status, TGVKV_STATUS_BUDGET);
+        if (n_active == 0) break;
+    }
+    if (has && budgets) budgets[lane] = result;
+}
+
 }  // namespace tgvkv

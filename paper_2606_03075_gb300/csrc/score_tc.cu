@@ -936,24 +936,52 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
     __syncthreads();
     if (s.cta_last) {
         __threadfence();
+        // the now idle K ring as scratch: the per-head masses, then the statistic
+        float* hs = reinterpret_cast<float*>(&s.k[0][0][0]);
+        const int units = p.head_budgets ? LH : p.L;
+        float* us = hs + LH;
+        // (the masses and the statistic take the ring's first half, the block
+        // split's scratch the second; larger problems read global memory)
+        const bool in_smem = (size_t)(LH + units) * sizeof(float) <= sizeof(s.k) / 2;
+        // every thread loads its share of the per-head masses (one round trip)
+        for (int lh = tid; lh < LH; lh += NTHREADS) {
+            const float a = __ldcg(&stat_head[lh]);
+            if (in_smem) hs[lh] = a;
+        }
+        __syncthreads();
         if (p.head_budgets) {
             // head-adaptive budgets: the statistic is the TV mass of each (layer, KV head)
-            for (int lh = tid; lh < p.L * p.H_kv; lh += NTHREADS) tvb_stat[lh] = __ldcg(&stat_head[lh]);
+            for (int lh = tid; lh < LH; lh += NTHREADS) {
+                const float a = in_smem ? hs[lh] : __ldcg(&stat_head[lh]);
+                tvb_stat[lh] = a;
+                if (in_smem) us[lh] = a;
+            }
         } else {
+            // each layer's masses added in head order
             for (int l = tid; l < p.L; l += NTHREADS) {
                 float S = 0.f;
-                for (int g = 0; g < p.H_kv; ++g) S += __ldcg(&stat_head[(size_t)l * p.H_kv + g]);
+                for (int g = 0; g < p.H_kv; ++g)
+                    S += in_smem ? hs[(size_t)l * p.H_kv + g] : __ldcg(&stat_head[(size_t)l * p.H_kv + g]);
                 tvb_stat[l] = S;
+                if (in_smem) us[l] = S;
             }
         }
+        __syncthreads();
         if (budgets) {
-            // the budgets of Eq. 5, with the now idle K ring as scratch
-            __syncthreads();
-            static_assert(sizeof(BudgetScratch) <= sizeof(s.k), "budget scratch in the K ring");
-            tvb_budget_block(tvb_stat, p.head_budgets ? p.L * p.H_kv : p.L, budget_total,
-                             p.basis == TGVKV_BASIS_ALL ? p.N : p.N_v,
-                             budgets, status, *reinterpret_cast<BudgetScratch*>(&s.k[0][0][0]),
-                             p.budget_stat == TGVKV_STAT_UNIFORM);
+            // the budgets of Eq. 5: one warp for up to 32 units, else the whole CTA
+            const int cap = p.basis == TGVKV_BASIS_ALL ? p.N : p.N_v;
+            const bool uniform = p.budget_stat == TGVKV_STAT_UNIFORM;
+            if (units <= 32 && in_smem) {
+                if (warp == 0)
+                    tvb_budget_warp(lane < units ? us[lane] : 0.f, units, budget_total, cap, budgets,
+                                    status, uniform, lane);
+            } else {
+                static_assert(sizeof(BudgetScratch) <= sizeof(s.k) / 2, "budget scratch in the K ring");
+                tvb_budget_block(tvb_stat, units, budget_total, cap, budgets, status,
+                                 *reinterpret_cast<BudgetScratch*>(reinterpret_cast<char*>(&s.k[0][0][0]) +
+                                                                   sizeof(s.k) / 2),
+                                 uniform);
+            }
         }
         if (tid == 0) *exit_counter = 0u;
     }
