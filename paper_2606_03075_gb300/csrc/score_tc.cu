@@ -934,6 +934,10 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
         s.cta_last = atomicAdd(exit_counter, 1u) == gridDim.x - 1;
     }
     __syncthreads();
+    // this CTA's scores and masses are written: a programmatic dependent (the
+    // select + gather of tgvkv_evict) may be scheduled once every CTA is here,
+    // while the last one still splits the budgets
+    griddep_launch_dependents();
     if (s.cta_last) {
         __threadfence();
         // the now idle K ring as scratch: the per-head masses, then the statistic

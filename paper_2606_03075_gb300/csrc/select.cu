@@ -159,7 +159,15 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
     __shared__ int span_red[64];
 
     for (int j = tid; j < p.N; j += kThreads) modality[j] = __ldg(modality_g + j);
-    int b = budgets[l];
+    __syncthreads();
+    int vlo = 0, vhi = 0;   // edge rows: positions [0, vlo) and [vhi, N)
+    if (COMPACT) vision_span_block(modality, p.N, &vlo, &vhi, span_red);
+    if (vhi < vlo) vhi = vlo;   // no vision key: every row is a leading edge row
+    // the scores and budgets come from the kernel before (as a programmatic
+    // dependent of the score kernel, this CTA may have started while its last
+    // CTA split the budgets): wait, then read them through L2
+    griddep_wait();
+    int b = __ldcg(budgets + l);
     if (b < 0 || b > p.N_v) {
         if (tid == 0) raise_status(status, TGVKV_STATUS_BUDGET);
         b = b < 0 ? 0 : p.N_v;
@@ -171,7 +179,7 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
     {
         long long part = 0;
         for (int m = tid; m < l; m += kThreads) {
-            int bm = budgets[m];
+            int bm = __ldcg(budgets + m);
             bm = bm < 0 ? 0 : (bm > p.N_v ? p.N_v : bm);
             part += (long long)p.H_kv * (p.N_t + bm);
         }
@@ -189,9 +197,6 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
     };
     // a set that would end past the caller's rows writes none of its rows or indices
     const bool fits = set_offset() + len <= capacity;
-    int vlo = 0, vhi = 0;   // edge rows: positions [0, vlo) and [vhi, N)
-    if (COMPACT) vision_span_block(modality, p.N, &vlo, &vhi, span_red);
-    if (vhi < vlo) vhi = vlo;   // no vision key: every row is a leading edge row
     if (edge_cta) {
         if (!fits) return;
         const long long off = set_offset();
@@ -210,7 +215,7 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
     }
     if (!fits) return;
     const float* sc = scores + (size_t)lg * p.N_v;
-    for (int i = tid; i < p.N_v; i += kThreads) keys[i] = float_order_key(__ldg(sc + i));
+    for (int i = tid; i < p.N_v; i += kThreads) keys[i] = float_order_key(__ldcg(sc + i));
     __syncthreads();
 
     // ---- radix select of the b-th largest key
@@ -429,13 +434,15 @@ tpr_select_warp_kernel(Problem p, const float* __restrict__ scores,
     int vlo, vhi;
     vision_span_block(modality, p.N, &vlo, &vhi, span_red);
     if (vhi < vlo) vhi = vlo;
+    // the scores and budgets come from the kernel before: wait, then read them through L2
+    griddep_wait();
     const bool edge_cta = blockIdx.x & 1;
     const int lg = (int)(blockIdx.x >> 1) * nw + wid;
     if (lg >= p.L * p.H_kv) return;
     const int l = lg / p.H_kv, g = lg % p.H_kv;
     const uint32_t lt = (1u << lane) - 1u;
 
-    int b = budgets[l];
+    int b = __ldcg(budgets + l);
     if (b < 0 || b > p.N_v) {
         if (lane == 0) raise_status(status, TGVKV_STATUS_BUDGET);
         b = b < 0 ? 0 : p.N_v;
@@ -444,7 +451,7 @@ tpr_select_warp_kernel(Problem p, const float* __restrict__ scores,
     // CSR offset: rows of every (layer, head) before this one
     long long off = 0;
     for (int m = lane; m < l; m += 32) {
-        int bm = budgets[m];
+        int bm = __ldcg(budgets + m);
         bm = bm < 0 ? 0 : (bm > p.N_v ? p.N_v : bm);
         off += (long long)p.H_kv * (p.N_t + bm);
     }
@@ -470,7 +477,7 @@ tpr_select_warp_kernel(Problem p, const float* __restrict__ scores,
     }
     if (!fits) return;
     const float* sc = scores + (size_t)lg * p.N_v;
-    for (int i = lane; i < p.N_v; i += 32) keys[i] = float_order_key(__ldg(sc + i));
+    for (int i = lane; i < p.N_v; i += 32) keys[i] = float_order_key(__ldcg(sc + i));
     __syncwarp();
 
     // ---- radix select of the b-th largest key, 8 bits per round
@@ -911,11 +918,11 @@ cudaError_t launch_sel_warp(const Problem& p, int nw, const float* scores, const
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const int heads = p.L * p.H_kv;
-    kern<<<2 * ((heads + nw - 1) / nw), nw * 32, smem, stream>>>(
-        p, scores, budgets, modality, offsets, idx, reinterpret_cast<const uint4*>(k),
-        reinterpret_cast<const uint4*>(v), reinterpret_cast<uint4*>(k_out),
-        reinterpret_cast<uint4*>(v_out), capacity, status);
-    return cudaGetLastError();
+    // a programmatic dependent of the kernel before (the score kernel on the evict path)
+    return launch_dependent(kern, dim3(2 * ((heads + nw - 1) / nw)), dim3(nw * 32), smem, stream, p,
+                            scores, budgets, modality, offsets, idx, reinterpret_cast<const uint4*>(k),
+                            reinterpret_cast<const uint4*>(v), reinterpret_cast<uint4*>(k_out),
+                            reinterpret_cast<uint4*>(v_out), capacity, status);
 }
 
 template <bool COMPACT, int VPR>
@@ -927,7 +934,13 @@ cudaError_t launch_sel(const Problem& p, const float* scores, const int32_t* bud
     const size_t smem = select_smem(p, COMPACT);
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    kern<<<p.L * p.H_kv * (COMPACT ? 2 : 1), kThreads, smem, stream>>>(
+    const dim3 grid(p.L * p.H_kv * (COMPACT ? 2 : 1));
+    if (COMPACT)   // a programmatic dependent of the kernel before (the score kernel on the evict path)
+        return launch_dependent(kern, grid, dim3(kThreads), smem, stream, p, scores, budgets, modality,
+                                offsets, idx, reinterpret_cast<const uint4*>(k),
+                                reinterpret_cast<const uint4*>(v), reinterpret_cast<uint4*>(k_out),
+                                reinterpret_cast<uint4*>(v_out), capacity, status);
+    kern<<<grid, kThreads, smem, stream>>>(
         p, scores, budgets, modality, offsets, idx,
         reinterpret_cast<const uint4*>(k),
         reinterpret_cast<const uint4*>(v), reinterpret_cast<uint4*>(k_out),
