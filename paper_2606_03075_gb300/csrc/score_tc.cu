@@ -590,6 +590,11 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constan
 
     // ------------------------------------------------------------ softmax
     if (warp >= 2 && warp < MMA2_WARP) {
+        // The kernel before (the select + gather of the previous eviction, when it
+        // is one) may still read the scores and budgets this kernel overwrites: the
+        // softmax role, the only one writing global memory before the end, waits
+        // for it.  The loads and MMAs of the first items overlap its end.
+        griddep_wait();
         const int sid = tid - 64;
         const int quarter = warp & 3;
         const int wi = (warp - 2) >> 2;                     // 0..3 within the lane quarter
@@ -1044,12 +1049,14 @@ cudaError_t launch_mode(const CUtensorMap& mq, const CUtensorMap& mk, const Prob
     const int sms = sm_count();
     if (sms <= 0) return cudaErrorInvalidDevice;
     const int grid = n_items < sms ? n_items : sms;
-    score_tc_kernel<D, MODE><<<grid, NTHREADS, smem, stream>>>(
-        mq, mk, p, n_items, n_two, modality, text_pos, w, scores, tvb_stat,
-        reinterpret_cast<float*>(ws + lay.score_part), reinterpret_cast<float*>(ws + lay.stat_part),
-        reinterpret_cast<float*>(ws + lay.stat_head), reinterpret_cast<uint32_t*>(ws + lay.tickets),
-        reinterpret_cast<uint32_t*>(ws + lay.status), budget_total, budgets);
-    return cudaGetLastError();
+    // a programmatic dependent of the kernel before (it may begin while that one ends)
+    return launch_dependent(score_tc_kernel<D, MODE>, dim3(grid), dim3(NTHREADS), smem, stream, mq, mk,
+                            p, n_items, n_two, modality, text_pos, w, scores, tvb_stat,
+                            reinterpret_cast<float*>(ws + lay.score_part),
+                            reinterpret_cast<float*>(ws + lay.stat_part),
+                            reinterpret_cast<float*>(ws + lay.stat_head),
+                            reinterpret_cast<uint32_t*>(ws + lay.tickets),
+                            reinterpret_cast<uint32_t*>(ws + lay.status), budget_total, budgets);
 }
 
 template <int D>

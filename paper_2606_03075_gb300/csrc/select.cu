@@ -150,6 +150,9 @@ tpr_select_kernel(Problem p, const float* __restrict__ scores, const int32_t* __
     __shared__ int s_kk;
     __shared__ int s_ties;
 
+    // a kernel after this one (the next eviction's score kernel) reads nothing
+    // this one writes: it may be scheduled once every CTA of this grid has begun
+    if (COMPACT) griddep_launch_dependents();
     // fused form: CTA 2h selects head h and gathers its interior rows, CTA
     // 2h + 1 copies its edge rows
     const int lg = COMPACT ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
@@ -421,6 +424,9 @@ tpr_select_warp_kernel(Problem p, const float* __restrict__ scores,
     extern __shared__ __align__(16) unsigned char dyn_raw[];
     const int wid = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nw = blockDim.x >> 5;
+    // a kernel after this one (the next eviction's score kernel) reads nothing
+    // this one writes: it may be scheduled once every CTA of this grid has begun
+    griddep_launch_dependents();
     const size_t mod_bytes = ((size_t)p.N + 15) & ~size_t(15);
     uint8_t* modality = dyn_raw;
     uint32_t* keys = reinterpret_cast<uint32_t*>(dyn_raw + mod_bytes) + (size_t)wid * warp_select_words(p);
