@@ -128,7 +128,19 @@ typedef struct tgvkv_desc {
                                then hold L * H_kv entries (head-major within a layer) */
 } tgvkv_desc;
 
-/* Bytes of device workspace the calls below need for this problem. */
+/* Size limits.  Every call checks the descriptor first and returns
+ * TGVKV_ERR_UNSUPPORTED, launching nothing, when a limit is exceeded:
+ *   N <= 32768 key positions per KV head (the score kernel holds a head's
+ *     per-tile vision tables in shared memory);
+ *   L <= 1024 layers;
+ *   G * n_win <= 32768 query rows per KV head;
+ *   L * H_kv <= 65535 KV heads in all (with head_budgets: <= 1024);
+ *   d = 64 or 128.
+ * TGVKV_ERR_INVALID_ARG covers the rest: non-positive L, H_q, H_kv or N,
+ * N_v outside [0, N], n_win < 0, H_q not a multiple of H_kv, an unknown mode. */
+
+/* Bytes of device workspace the calls below need for this problem (0 when the
+ * descriptor is rejected). */
 size_t tgvkv_workspace_size(const tgvkv_desc* desc);
 
 /* B_V = floor(ratio * N_v * L + 1/2): vision rows kept per KV head over all

@@ -76,6 +76,31 @@ def test_validation_rejects_before_launch(lib):
     assert lib.tgvkv_status(None, None) < 0
 
 
+def test_descriptor_limits(lib):
+    """The size limits include/tgvkv.h states, at and just past each bound
+    (tgvkv_workspace_size is 0 exactly when a descriptor is rejected)."""
+    def ws(**kw):
+        return lib.tgvkv_workspace_size(ctypes.byref(_desc(**kw)))
+
+    assert ws(N=32768, N_v=32600) > 0
+    assert ws(N=32769, N_v=32600) == 0
+    assert ws(L=1024) > 0
+    assert ws(L=1025) == 0
+    assert ws(H_q=256, H_kv=1, n_win=128, w_layer_stride=128) > 0      # G * n_win = 32768
+    assert ws(H_q=257, H_kv=1, n_win=128, w_layer_stride=128) == 0
+    assert ws(L=255, H_q=257, H_kv=257) > 0                            # L * H_kv = 65535
+    assert ws(L=256, H_q=256, H_kv=256) == 0
+    assert ws(L=32, H_q=32, H_kv=32, head_budgets=1) > 0               # 1024 heads
+    assert ws(L=33, H_q=32, H_kv=32, head_budgets=1) == 0
+    assert ws(d=64) > 0 and ws(d=128) > 0
+    for bad in (dict(d=32), dict(d=256), dict(L=0), dict(H_kv=0), dict(N=0), dict(N_v=-1),
+                dict(N_v=101), dict(n_win=-1), dict(H_q=6, H_kv=4), dict(budget_basis=2),
+                dict(weight_mode=2), dict(budget_stat=3), dict(head_budgets=2),
+                dict(keep_first=-1), dict(head_budgets=1, budget_stat=1)):
+        assert ws(**bad) == 0, bad
+    assert ws(n_win=0) > 0 and ws(N_v=0) > 0 and ws(N_v=100) > 0
+
+
 def test_host_budget_arithmetic_matches_oracle(lib):
     ref = ctypes.byref
     for name, wl in synth.WORKLOADS.items():

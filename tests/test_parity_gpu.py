@@ -130,6 +130,19 @@ def test_small_layouts(api, name):
         _full_check(api, wl, r)
 
 
+def test_max_length_heads(api):
+    """Heads of the largest length the library accepts (N = 32768): the score
+    kernel's per-head tile tables at their full size, text before and after the
+    vision span, G = 2, and the select + gather in its two-launch form (its
+    shared-memory tables exceed the fused kernel's at this length)."""
+    wl = synth.custom("max_len", 1, 4, 2, 128,
+                      [("text", 40), ("vision", 32600), ("text", 128)], window=64,
+                      ratios=(0.05,))
+    assert wl.N == 32768
+    assert api.tgvkv_evict_launches(api.desc_for_workload(wl)) == 3
+    _full_check(api, wl, 0.05)
+
+
 @pytest.mark.parametrize("name", sorted(ONE_TILE))
 def test_one_tile_layouts(api, name):
     """The whole step against the oracle, then the score call alone (scores
