@@ -143,6 +143,28 @@ def test_max_length_heads(api):
     _full_check(api, wl, 0.05)
 
 
+def test_max_layers(api):
+    """The most layers the library accepts (L = 1024): the score kernel's
+    closing CTA sums 1024 layer masses and splits the budgets with the whole
+    block (more than one warp's worth of units), and the warp-per-head select
+    + gather runs 1024 sets."""
+    wl = synth.custom("max_layers", 1024, 2, 1, 64,
+                      [("text", 8), ("vision", 120), ("text", 16)], window=16, ratios=(0.1,))
+    assert api.tgvkv_evict_launches(api.desc_for_workload(wl)) == 2
+    _full_check(api, wl, 0.1)
+
+
+def test_max_query_rows(api):
+    """The most query rows per KV head the library accepts (G * n_win = 32768,
+    256 row tiles of one head): every row tile's partial scores summed into
+    the head's."""
+    wl = synth.custom("max_rows", 1, 256, 1, 64,
+                      [("text", 64), ("vision", 256), ("text", 128)], window=128,
+                      ratios=(0.2,))
+    assert wl.H_q // wl.H_kv * wl.n_win == 32768
+    _full_check(api, wl, 0.2)
+
+
 @pytest.mark.parametrize("name", sorted(ONE_TILE))
 def test_one_tile_layouts(api, name):
     """The whole step against the oracle, then the score call alone (scores
