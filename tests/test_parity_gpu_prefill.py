@@ -354,6 +354,47 @@ def test_full_size_long_prefill_then_evict(api, name, ratio, layer, n_prefix):
     P.check_selection_and_compaction(wl, inp, g, [layer], ref_scores=ref_s)
 
 
+def test_prefill_max_length(api):
+    """Heads of the largest length the library accepts (N = 32768): the
+    prefill's per-tile tables at their full size.  The first 512 rows against
+    the oracle on the truncated sequence (exact for causal rows), the last row
+    (which sees every key) against the oracle's attention over all of them,
+    the query rows' statistics over all keys, then the eviction with them."""
+    wl = synth.custom("max_len_prefill", 1, 2, 1, 64,
+                      [("text", 40), ("vision", 32600), ("text", 128)], window=64,
+                      ratios=(0.05,))
+    assert wl.N == 32768
+    inp = synth.generate_prefill(wl, seed=0)
+    dev = P.device_inputs(inp)
+    o, q_text, stats = _run_prefill(api, wl, inp, dev)
+    scale = 1.0 / math.sqrt(wl.d)
+    q1, k1, v1 = (oracle.widen_bf16(inp[n]) for n in ("q_all", "k", "v"))
+    o_gpu = oracle.widen_bf16(o.view(torch.int16).cpu().numpy())
+    n_prefix = 512
+    o_ref, bound = oracle.prefill_attention(q1[:, :, :n_prefix], k1[:, :, :n_prefix],
+                                            v1[:, :, :n_prefix], scale, wl.H_kv)
+    assert np.all(np.abs(o_gpu[:, :, :n_prefix] - o_ref) <= 2.0 ** -7 * bound + 1e-6)
+    # the last row: attention over the whole sequence, as one set of every row
+    last, every = wl.N - 1, np.array([0, wl.N])
+    o_last = oracle.decode_attention(q1[:, :, last], k1[0, 0], v1[0, 0], every, wl.H_kv, scale)
+    b_last = oracle.decode_attention(q1[:, :, last], k1[0, 0], np.abs(v1[0, 0]), every, wl.H_kv,
+                                     scale)
+    assert np.all(np.abs(o_gpu[:, :, last] - o_last) <= 2.0 ** -7 * b_last + 1e-6)
+    np.testing.assert_array_equal(q_text.view(torch.int16).cpu().numpy(), inp["q"])
+    lse2, vis = oracle.row_statistics(q1, k1, inp["modality"], inp["text_pos"], scale, wl.H_kv)
+    st = stats.cpu().numpy().astype(np.float64)
+    assert np.all(np.abs(st[..., 0] + np.log2(st[..., 1]) - lse2) <= 1e-3)
+    P.assert_close(st[..., 2] / st[..., 1], vis, "vision share")
+    g = _run_evict_with_stats(api, wl, dev, q_text, stats, 0.05)
+    assert g["status"] == 0
+    ref_s, ref_t = P.oracle_scores(wl, inp, [0])
+    P.assert_close(g["scores"], ref_s, "scores")
+    P.assert_close(g["stat"], ref_t, "tvb_stat")
+    total = oracle.vision_budget_total(0.05, wl.N_v, wl.L)
+    assert g["budgets"].tolist() == [total]
+    P.check_selection_and_compaction(wl, inp, g, [0], ref_scores=ref_s)
+
+
 @pytest.mark.parametrize("stat", ["tv", "uniform"])
 def test_evict_with_statistics_head_budgets(api, stat):
     """Head-adaptive budgets with given statistics: the per-head TV masses come
