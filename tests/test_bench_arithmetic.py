@@ -35,3 +35,19 @@ def test_score_flops_and_exponentials_by_counting_pairs():
     assert bench.score_flops(wl) == 2 * wl.d * wl.L * wl.H_q * visible
     assert bench.score_exps(wl) == wl.L * wl.H_q * (visible + visible_vision)
     assert np.all(np.diff(pos) > 0)
+
+
+def test_clock_rule_rejects_slowdowns_and_stuck_clocks():
+    """The timing rule on clocks: a hardware or thermal slowdown, or a median
+    SM clock well below the maximum with no reason given, disqualifies a timed
+    region; the power cap alone does not, nor does a missing NVML."""
+    ok = dict(sm_mhz=2070, sm_max_mhz=2070, reasons=[])
+    assert not bench.clocks_rejected(ok)
+    assert not bench.clocks_rejected(dict(ok, sm_mhz=1800, reasons=["sw_power_cap"]))
+    assert not bench.clocks_rejected(dict(ok, sm_mhz=1200, reasons=["sw_power_cap"]))
+    for r in ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown"):
+        assert bench.clocks_rejected(dict(ok, reasons=[r]))
+        assert bench.clocks_rejected(dict(ok, reasons=["sw_power_cap", r]))
+    assert bench.clocks_rejected(dict(ok, sm_mhz=1500))          # locked low, no reason
+    assert not bench.clocks_rejected(dict(ok, sm_mhz=1700))      # 82% of the maximum
+    assert not bench.clocks_rejected(dict(sm_mhz=None, sm_max_mhz=None, reasons=[]))
