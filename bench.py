@@ -1030,7 +1030,8 @@ def main():
                                             "rows read, idx and offsets"},
             "roofline": {"bound": roof["bound"], "kernel": dom, "achieved": roof["achieved"],
                          "peak": roof["peak"], "unit": roof["unit"], "frac": roof["frac"],
-                         "traffic": traffic, "bytes_per_launch": roof["bytes_per_launch"],
+                         "traffic": traffic, "source_sha": source_hash(dom),
+                         "bytes_per_launch": roof["bytes_per_launch"],
                          "flops_per_launch": roof["flops_per_launch"],
                          "launch_ms": stage_ms[dom],
                          "peak_source": roof["peak_source"], "frac_nominal": roof["frac_nominal"]},
