@@ -803,3 +803,103 @@ def test_row_statistics_closed_form_and_eq5():
     l, h, i = 1, 4, 2
     x = [0.6 * float(q[l, h, i] @ k[l, h // 3, j]) for j in range(pos[i] + 1)]
     assert abs(lse2[l, h, i] - math.log2(sum(math.exp(t) for t in x))) < 1e-12
+
+
+# ---------------------------------------------------------------- edges found by planting mistakes
+def test_budget_totals_round_half_up_exact():
+    """B_V and B are the nearest integer to r N L with halves rounded up,
+    checked in exact rational arithmetic on ratios that are binary fractions
+    (so r N L is exact in floating point): fractional parts 0, 1/4, 1/2, 3/4."""
+    from fractions import Fraction
+    for r, n, L in [(0.25, 6, 1), (0.25, 5, 1), (0.25, 7, 1), (0.125, 4, 1), (0.375, 2, 1),
+                    (0.0, 100, 32), (1.0, 37, 3), (0.0625, 72, 3), (0.5, 3, 3)]:
+        want = math.floor(Fraction(r) * n * L + Fraction(1, 2))
+        assert oracle.vision_budget_total(r, n, L) == want, (r, n, L)
+        assert oracle.all_budget_total(r, n, L) == want, (r, n, L)
+
+
+def test_tvb_budget_zero_total_and_layer_exactly_at_cap():
+    """A zero total gives zero budgets.  Eq. 5 with stat (3, 1, 5), total 4,
+    cap 2, by hand: quotas 4*3/9 = 1.333, 4*1/9 = 0.444, 4*5/9 = 2.222; floors
+    1, 0, 2 leave one unit, which goes to the largest fraction (layer 1):
+    (1, 1, 2).  Layer 2 sits exactly at the cap, which does not exceed it, so
+    nothing is re-split (re-splitting would give (2, 0, 2))."""
+    assert oracle.tvb_budgets([0.3, 0.5, 0.2], 0, 10) == [0, 0, 0]
+    assert oracle.tvb_budgets([3.0, 1.0, 5.0], 4, 2) == [1, 1, 2]
+
+
+def test_sink_positions_by_hand():
+    """The first keep_first and last keep_last positions, clipped to the
+    sequence, as a sorted set."""
+    assert oracle.sink_positions(10, 2, 3).tolist() == [0, 1, 7, 8, 9]
+    assert oracle.sink_positions(5, 0, 0).tolist() == []
+    assert oracle.sink_positions(4, 3, 3).tolist() == [0, 1, 2, 3]
+    assert oracle.sink_positions(3, 0, 5).tolist() == [0, 1, 2]
+    assert oracle.sink_positions(3, 5, 0).tolist() == [0, 1, 2]
+    assert oracle.sink_positions(6, 0, 1).tolist() == [5]
+
+
+def test_selection_without_sinks_by_default():
+    """With default arguments neither the general selection nor the whole step
+    keeps sinks: on a layout whose first and last tokens are vision keys with
+    the lowest scores, the kept vision keys are exactly the top b by (score
+    descending, position ascending), found by a plain sort."""
+    modality = np.array([1, 1, 0, 1, 1, 1, 0, 0, 1, 1], np.uint8)
+    vision = np.flatnonzero(modality == 1)
+    text = np.flatnonzero(modality == 0)
+    scores = np.array([[[0.01, 0.5, 0.4, 0.9, 0.3, 0.2, 0.02]]])
+    for b in (1, 3, 5):
+        _, idx = oracle.tpr_select_general(scores, None, [b], modality, vision_basis=True)
+        top = sorted(range(vision.size), key=lambda i: (-scores[0, 0, i], i))[:b]
+        assert idx.tolist() == sorted(text.tolist() + vision[top].tolist())
+    # the whole step on such a layout: q and k random, the first and last
+    # tokens vision; the kept vision keys per head are the top b_l of its scores
+    rng = np.random.default_rng(7)
+    L, H, d = 2, 2, 8
+    modality = np.array([1, 1, 1, 0, 0, 1, 1, 1, 0, 0, 0, 1], np.uint8)
+    pos = np.array([8, 9, 10])
+    q = synth.to_bf16_bits(rng.standard_normal((L, H, pos.size, d)))
+    k = synth.to_bf16_bits(rng.standard_normal((L, H, modality.size, d)))
+    v = synth.to_bf16_bits(rng.standard_normal((L, H, modality.size, d)))
+    w = np.full((L, pos.size), 1.0 / pos.size)
+    ref = oracle.evict(q, k, v, modality, pos, w, 0.4, H)
+    vision = np.flatnonzero(modality == 1)
+    for l in range(L):
+        for g in range(H):
+            rows = ref["idx"][ref["offsets"][l * H + g]:ref["offsets"][l * H + g + 1]]
+            s = ref["scores"][l, g]
+            top = sorted(range(vision.size), key=lambda i: (-s[i], i))[:int(ref["budgets"][l])]
+            assert sorted(set(rows.tolist()) & set(vision.tolist())) == sorted(vision[top].tolist())
+
+
+def test_no_sets_for_no_layers():
+    """Zero layers give one offset (0) and no indices."""
+    modality = np.array([0, 1, 1, 0], np.uint8)
+    off, idx = oracle.tpr_select(np.zeros((0, 2, 2)), [], modality)
+    assert off.tolist() == [0] and idx.size == 0
+    off, idx = oracle.tpr_select_general(np.zeros((0, 2, 2)), None, [], modality,
+                                         vision_basis=True)
+    assert off.tolist() == [0] and idx.size == 0
+
+
+def test_attention_saturates_without_overflow():
+    """Logits in the thousands: each softmax row is one-hot on its largest
+    logit (the others are e^-1000 or less below it), so the decode output and
+    every prefill row equal that key's value row exactly, with no overflow."""
+    d, n = 4, 4
+    k = np.eye(n, d)[None, None] * 1.0                      # orthonormal keys
+    v = np.arange(n * d, dtype=np.float64).reshape(1, 1, n, d) + 1.0
+    q = 1000.0 * k[:, :, ::-1].copy()                       # row i aims at key n-1-i
+    o, bound = oracle.prefill_attention(q, k, v, 1.0, 1)
+    for i in range(n):
+        visible = np.arange(i + 1)
+        logits = [1000.0 if j == n - 1 - i else 0.0 for j in visible]
+        if max(logits) == 0.0:
+            want = v[0, 0, :i + 1].mean(axis=0)               # all visible logits equal
+        else:
+            want = v[0, 0, n - 1 - i]
+        np.testing.assert_allclose(o[0, 0, i], want, rtol=0, atol=1e-12)
+    out = oracle.decode_attention(q[:, :, 0], k[0, 0], v[0, 0], np.array([0, n]), 1, 1.0)
+    np.testing.assert_allclose(out[0, 0], v[0, 0, n - 1], rtol=0, atol=1e-12)
+    out = oracle.decode_attention(-q[:, :, 0], k[0, 0], v[0, 0], np.array([0, n]), 1, 1.0)
+    np.testing.assert_allclose(out[0, 0], v[0, 0, :n - 1].mean(axis=0), rtol=0, atol=1e-12)
