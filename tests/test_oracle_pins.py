@@ -903,3 +903,36 @@ def test_attention_saturates_without_overflow():
     np.testing.assert_allclose(out[0, 0], v[0, 0, n - 1], rtol=0, atol=1e-12)
     out = oracle.decode_attention(-q[:, :, 0], k[0, 0], v[0, 0], np.array([0, n]), 1, 1.0)
     np.testing.assert_allclose(out[0, 0], v[0, 0, :n - 1].mean(axis=0), rtol=0, atol=1e-12)
+
+
+def test_evict_one_sided_sinks_and_row_wiring():
+    """The whole step with only first-token or only last-token sinks (vision
+    basis), on a layout whose first and last tokens are vision keys: the sink
+    is kept and takes one of the head's b_l vision slots, the other b_l - 1
+    slots go to the top scores of the remaining vision keys (a plain sort);
+    k_out / v_out hold the K / V rows of the kept positions (direct indexing)."""
+    rng = np.random.default_rng(11)
+    L, H, d = 2, 2, 8
+    modality = np.array([1, 1, 1, 0, 0, 1, 1, 1, 0, 0, 0, 1], np.uint8)
+    pos = np.array([8, 9, 10])
+    q = synth.to_bf16_bits(rng.standard_normal((L, H, pos.size, d)))
+    k = synth.to_bf16_bits(rng.standard_normal((L, H, modality.size, d)))
+    v = synth.to_bf16_bits(rng.standard_normal((L, H, modality.size, d)))
+    w = np.full((L, pos.size), 1.0 / pos.size)
+    vision = np.flatnonzero(modality == 1)
+    for first, last in ((1, 0), (0, 1)):
+        sink = 0 if first else modality.size - 1
+        ref = oracle.evict(q, k, v, modality, pos, w, 0.4, H, keep_first=first, keep_last=last)
+        for l in range(L):
+            b = int(ref["budgets"][l])
+            assert b >= 1
+            for g in range(H):
+                lo, hi = ref["offsets"][l * H + g], ref["offsets"][l * H + g + 1]
+                rows = ref["idx"][lo:hi]
+                s = ref["scores"][l, g]
+                rest = [i for i in range(vision.size) if vision[i] != sink]
+                top = sorted(rest, key=lambda i: (-s[i], i))[:b - 1]
+                want = sorted([sink] + vision[top].tolist())
+                assert sorted(set(rows.tolist()) & set(vision.tolist())) == want, (first, l, g)
+                np.testing.assert_array_equal(ref["k_out"][lo:hi], k[l, g][rows])
+                np.testing.assert_array_equal(ref["v_out"][lo:hi], v[l, g][rows])
