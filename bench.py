@@ -178,10 +178,11 @@ def score_flops(wl):
 
 # each kernel's source with the headers it includes (a change to any of them
 # invalidates a recorded ncu traffic figure)
-KERNEL_SOURCES = {"score": ("score_tc.cu", "rowstat.cuh", "tc05.cuh", "common.cuh"),
+KERNEL_SOURCES = {"score": ("score_tc.cu", "budget.cuh", "rowstat.cuh", "tc05.cuh", "common.cuh"),
                   "budget": ("budget.cu", "budget.cuh", "common.cuh"),
-                  "select": ("select.cu", "budget.cuh", "common.cuh"),
-                  "compact": ("compact.cu", "common.cuh")}
+                  "select": ("select.cu", "common.cuh"),
+                  "compact": ("compact.cu", "common.cuh"),
+                  "tail": ("select.cu", "compact.cu", "common.cuh")}
 
 
 def source_hash(stage):

@@ -51,3 +51,25 @@ def test_clock_rule_rejects_slowdowns_and_stuck_clocks():
     assert bench.clocks_rejected(dict(ok, sm_mhz=1500))          # locked low, no reason
     assert not bench.clocks_rejected(dict(ok, sm_mhz=1700))      # 82% of the maximum
     assert not bench.clocks_rejected(dict(sm_mhz=None, sm_max_mhz=None, reasons=[]))
+
+
+def test_traffic_hash_covers_every_included_kernel_header():
+    """A recorded ncu traffic figure stays valid only while the kernel's source
+    is unchanged: each kernel's hash list must hold its .cu file and every
+    kernel header it includes, directly or through another header (launch.h
+    declares host launchers only)."""
+    import os
+    import re
+    csrc = os.path.join(os.path.dirname(bench.__file__), "paper_2606_03075_gb300", "csrc")
+
+    def local_includes(name, seen):
+        for inc in re.findall(r'#include "([^"]+)"', open(os.path.join(csrc, name)).read()):
+            if inc not in seen and os.path.exists(os.path.join(csrc, inc)):
+                seen.add(inc)
+                local_includes(inc, seen)
+        return seen
+
+    for stage, files in bench.KERNEL_SOURCES.items():
+        for cu in (f for f in files if f.endswith(".cu")):
+            missing = local_includes(cu, set()) - set(files) - {"launch.h"}
+            assert not missing, (stage, cu, missing)
