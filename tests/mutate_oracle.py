@@ -1,6 +1,11 @@
 """Mutation check of the oracle's pins (not collected by pytest; run by hand):
 
-    python tests/mutate_oracle.py [pytest args, default tests/test_oracle_pins.py]
+    python tests/mutate_oracle.py [--source FILE] [--funcs F1,F2] [pytest args,
+                                   default tests/test_oracle_pins.py]
+
+(--source picks another host-side file to mutate, e.g.
+paper_2606_03075_gb300/shard.py with tests/test_shard.py; --funcs keeps only
+the sites inside the named functions, e.g. bench.py's roofline arithmetic.)
 
 Plants one plausible mistake at a time in a copy of oracle/tgvkv_oracle.py
 (an operator or comparison swapped, a constant, index, slice bound or axis off
@@ -20,7 +25,7 @@ import tempfile
 import time
 
 REPO = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
-SRC = os.path.join(REPO, "oracle", "tgvkv_oracle.py")
+SRC = "oracle/tgvkv_oracle.py"
 
 SWAP_BIN = {ast.Add: ast.Sub, ast.Sub: ast.Add, ast.Mult: ast.Div, ast.Div: ast.Mult,
             ast.FloorDiv: ast.Div}
@@ -169,20 +174,22 @@ def mutate(tree, node, kind):
     raise ValueError(kind)
 
 
-def main(pytest_args):
+def main(pytest_args, src=SRC, funcs=None):
     work = tempfile.mkdtemp(prefix="tgvkv_mut_")
     try:
-        for d in ("tests", "oracle", "paper_2606_03075_gb300"):
+        for d in ("tests", "oracle", "paper_2606_03075_gb300", "profiles"):
             shutil.copytree(os.path.join(REPO, d), os.path.join(work, d),
                             ignore=shutil.ignore_patterns("*.so", "__pycache__", "_build*"))
-        shutil.copy(os.path.join(REPO, "pytest.ini"), work)
-        base = ast.parse(open(SRC).read())
+        for f in ("pytest.ini", "bench.py"):
+            shutil.copy(os.path.join(REPO, f), work)
+        base = ast.parse(open(os.path.join(REPO, src)).read())
         finder = Sites()
         finder.visit(base)
-        n = len(finder.sites)
+        chosen = [i for i, (_, _, f) in enumerate(finder.sites) if funcs is None or f in funcs]
+        n = len(chosen)
         print(f"{n} mutants", flush=True)
         survived, killed, t0 = 0, 0, time.time()
-        for i in range(n):
+        for i in chosen:
             tree = copy.deepcopy(base)
             walk = Sites()
             walk.visit(tree)
@@ -190,7 +197,7 @@ def main(pytest_args):
             line = node.lineno
             tree, what = mutate(tree, node, kind)
             ast.fix_missing_locations(tree)
-            with open(os.path.join(work, "oracle", "tgvkv_oracle.py"), "w") as f:
+            with open(os.path.join(work, src), "w") as f:
                 f.write(ast.unparse(tree))
             r = subprocess.run([sys.executable, "-m", "pytest", *pytest_args, "-x", "-q",
                                 "-p", "no:cacheprovider", "-m", "not gpu"],
@@ -206,4 +213,12 @@ def main(pytest_args):
 
 
 if __name__ == "__main__":
-    main(sys.argv[1:] or ["tests/test_oracle_pins.py"])
+    args = sys.argv[1:]
+    source, only = SRC, None
+    while args[:1] in (["--source"], ["--funcs"]):
+        if args[0] == "--source":
+            source = args[1]
+        else:
+            only = set(args[1].split(","))
+        args = args[2:]
+    main(args or ["tests/test_oracle_pins.py"], source, only)

@@ -73,3 +73,41 @@ def test_traffic_hash_covers_every_included_kernel_header():
         for cu in (f for f in files if f.endswith(".cu")):
             missing = local_includes(cu, set()) - set(files) - {"launch.h"}
             assert not missing, (stage, cu, missing)
+
+
+def test_roof_and_mufu_rate_by_hand():
+    """One layer, two query heads on one KV head, d = 64, 10 text + 100 vision +
+    18 text tokens with the last 18 (positions 110..127) as query rows.
+    Score launch bytes: K 128*64*2 = 16384, Q 2*18*64*2 = 4608, scores 100*4 =
+    400: 21392.  FLOPs: 2*64*2 * sum_{p=110..127}(p+1) = 256 * 2151 = 550656.
+    At 1000 GB/s and 1 TFLOP/s the FLOPs take longer (550.656 ns > 21.392 ns):
+    tensor-bound.  Exponentials: 2 heads * (2151 + 18*100) = 7902."""
+    import pytest
+    wl = synth.custom("hand", 1, 2, 1, 64, [("text", 10), ("vision", 100), ("text", 18)])
+    assert wl.text_pos.tolist() == list(range(110, 128))
+    peaks = {"hbm_gbs": 1000.0, "bf16_tflops": 1.0}
+    r = bench.kernel_roof(wl, 0.5, "score", 1.0, peaks)
+    assert r["bytes_per_launch"] == 21392 and r["flops_per_launch"] == 550656
+    assert r["bound"] == "tensor" and r["unit"] == "TFLOP/s" and r["peak"] == 1.0
+    assert r["achieved"] == pytest.approx(550656 / 1e-3 / 1e12)
+    assert r["frac"] == pytest.approx(550656 / 1e-3 / 1e12 / 1.0)
+    assert r["frac_nominal"] == pytest.approx(550656 / 1e-3 / 1e12 / 2250.0)
+    # a much slower tensor peak keeps it tensor-bound; a much faster one makes
+    # the bytes bind: 550656 / 1e15 s < 21392 / 1e12 s
+    r = bench.kernel_roof(wl, 0.5, "score", 2.0, {"hbm_gbs": 1000.0, "bf16_tflops": 1000.0})
+    assert r["bound"] == "hbm" and r["unit"] == "GB/s" and r["peak"] == 1000.0
+    assert r["achieved"] == pytest.approx(21392 / 2e-3 / 1e9)
+    assert r["frac"] == pytest.approx(21392 / 2e-3 / 1e9 / 1000.0)
+    assert r["frac_nominal"] == pytest.approx(21392 / 2e-3 / 1e9 / 7900.0)
+    # the fused tail has no FLOPs: HBM-bound on its bytes (scores read, kept
+    # rows read and written, idx, offsets); r = 0.5 keeps 18 + 10 text rows and
+    # B_V = floor(0.5 * 100 + 1/2) = 50 vision rows: 78 rows
+    tail = 400 + 4 * 78 * 64 * 2 + 4 * 78 + 8 * 2
+    assert bench.stage_bytes(wl, 0.5)["tail"] == tail
+    r = bench.kernel_roof(wl, 0.5, "tail", 1.0, peaks)
+    assert r["bound"] == "hbm" and r["flops_per_launch"] == 0 and r["bytes_per_launch"] == tail
+    m = bench.mufu_of(wl, 1.0, 2000.0)
+    assert m["exps_per_launch"] == 7902
+    assert m["peak_G_per_s"] == pytest.approx(32 * 152 * 2000e6 / 1e9)
+    assert m["achieved_G_per_s"] == pytest.approx(7902 / 1e-3 / 1e9)
+    assert m["frac"] == pytest.approx(7902 / 1e-3 / 1e9 / (32 * 152 * 2.0))
