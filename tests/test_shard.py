@@ -1,4 +1,4 @@
-"""Layer-sharded eviction on CPU ranks (gloo, world size 2): the host logic of
+"""Sharded eviction on CPU ranks (gloo, world size 2 and 3): the host logic of
 paper_2606_03075_gb300.shard -- layer ranges, the all-gather of the TVB
 statistic, identical budgets on every rank -- driven with the fp64 oracle as
 the compute backend, against the unsharded oracle."""
@@ -83,8 +83,10 @@ def test_layer_ranges_cover_every_layer_once():
         shard.layer_range(4, 2, 2)
 
 
-def test_two_cpu_ranks_match_the_unsharded_oracle():
-    world = 2
+@pytest.mark.parametrize("world", [2, 3])
+def test_cpu_ranks_match_the_unsharded_oracle(world):
+    """5 layers over 2 ranks (3 + 2) or 3 ranks (2 + 2 + 1): the statistic's
+    slices differ in length, so the all-gather's padding is exercised."""
     with tempfile.TemporaryDirectory() as outdir:
         mp.spawn(_rank_main, args=(world, _free_port(), outdir), nprocs=world, join=True)
         parts = [dict(np.load(os.path.join(outdir, f"r{r}.npz"))) for r in range(world)]
@@ -160,7 +162,7 @@ class OracleHeadBackend(OracleBackend):
         return torch.from_numpy(s), torch.from_numpy(np.asarray(m, np.float64))
 
 
-WLH = synth.custom("shard_heads", 3, 8, 4, 64, [("text", 9), ("vision", 70), ("text", 6),
+WLH = synth.custom("shard_heads", 3, 10, 5, 64, [("text", 9), ("vision", 70), ("text", 6),
                                                 ("vision", 30), ("text", 12)],
                    weights="dirichlet", ratios=(0.2,))
 
@@ -186,8 +188,10 @@ def _rank_heads(rank, world, port, outdir):
         dist.destroy_process_group()
 
 
-def test_two_cpu_ranks_sharded_by_kv_head_match_the_unsharded_oracle():
-    world = 2
+@pytest.mark.parametrize("world", [2, 3])
+def test_cpu_ranks_sharded_by_kv_head_match_the_unsharded_oracle(world):
+    """5 KV heads over 2 ranks (3 + 2) or 3 ranks (2 + 2 + 1): padded blocks in
+    the all-gather of the per-head masses."""
     inp = synth.generate(WLH, seed=9)
     ref = oracle.evict(inp["q"], inp["k"], inp["v"], inp["modality"], inp["text_pos"], inp["w"],
                        0.2, WLH.H_kv)
