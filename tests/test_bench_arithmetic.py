@@ -111,3 +111,53 @@ def test_roof_and_mufu_rate_by_hand():
     assert m["peak_G_per_s"] == pytest.approx(32 * 152 * 2000e6 / 1e9)
     assert m["achieved_G_per_s"] == pytest.approx(7902 / 1e-3 / 1e9)
     assert m["frac"] == pytest.approx(7902 / 1e-3 / 1e9 / (32 * 152 * 2.0))
+
+
+def test_stage_bytes_rounding_and_boundaries_by_hand():
+    """The same hand workload: every launch's algorithmic bytes, the budget
+    total's rounding (exact rationals), the roof choice just either side of the
+    point where bytes and FLOPs take equal time, rates at launch times other
+    than 1 ms, and the clock rule exactly at 80% of the maximum."""
+    import math as _m
+    from fractions import Fraction
+    import pytest
+    wl = synth.custom("hand", 1, 2, 1, 64, [("text", 10), ("vision", 100), ("text", 18)])
+    sb = bench.stage_bytes(wl, 0.5)
+    rows = 78                                   # 28 text + 50 vision rows, one KV head
+    assert bench.step_bytes(wl, 0.5) == (16384 + 2 * rows * 64 * 2, rows)
+    assert sb["budget"] == 8                    # one fp32 statistic read, one int32 budget written
+    assert sb["select"] == 400 + 4 * rows + 8 * 2          # scores, idx, offsets
+    assert sb["compact"] == 4 * rows * 64 * 2 + 4 * rows   # kept K/V read + written, idx read
+    assert sb["tail"] == 400 + 4 * rows * 64 * 2 + 4 * rows + 8 * 2
+    for r, nv, L in [(0.25, 6, 1), (0.25, 5, 1), (0.25, 7, 1), (0.125, 4, 1), (0.375, 2, 1)]:
+        w2 = synth.custom("r", L, 1, 1, 64, [("text", 1), ("vision", nv)])
+        assert bench.budget_total(w2, r) == _m.floor(Fraction(r) * nv * L + Fraction(1, 2))
+    # bytes take 21392 / 1e12 s = 21.392 ns at 1000 GB/s; the FLOPs take
+    # 550656 / (T * 1e12) s: 22.03 ns at T = 25 (tensor-bound), 20.78 ns at 26.5
+    assert bench.kernel_roof(wl, 0.5, "score", 0.25, {"hbm_gbs": 1000.0,
+                                                      "bf16_tflops": 25.0})["bound"] == "tensor"
+    r = bench.kernel_roof(wl, 0.5, "score", 0.25, {"hbm_gbs": 1000.0, "bf16_tflops": 26.5})
+    assert r["bound"] == "hbm"
+    assert r["achieved"] == pytest.approx(21392 / 0.25e-3 / 1e9)
+    r = bench.kernel_roof(wl, 0.5, "score", 0.25, {"hbm_gbs": 1000.0, "bf16_tflops": 25.0})
+    assert r["achieved"] == pytest.approx(550656 / 0.25e-3 / 1e12)
+    m = bench.mufu_of(wl, 0.5, 1000.0)
+    assert m["achieved_G_per_s"] == pytest.approx(7902 / 0.5e-3 / 1e9)
+    assert m["peak_G_per_s"] == pytest.approx(32 * 152 * 1.0)
+    # exactly 80% of the maximum is not "below 80%"
+    assert not bench.clocks_rejected(dict(sm_mhz=1656.0, sm_max_mhz=2070, reasons=[]))
+    assert bench.clocks_rejected(dict(sm_mhz=1655.0, sm_max_mhz=2070, reasons=[]))
+
+
+def test_stage_bytes_two_layers_two_kv_heads_by_hand():
+    """L = 2, H_kv = 2 (G = 2), 10 + 100 + 18 tokens, r = 0.5: B_V = floor(0.5 *
+    100 * 2 + 1/2) = 100, rows = 2 * (2 * 28 + 100) = 312, scores 2*2*100*4 =
+    1600 bytes, offsets 8 * (2*2 + 1) = 40 bytes."""
+    wl = synth.custom("hand2", 2, 4, 2, 64, [("text", 10), ("vision", 100), ("text", 18)])
+    sb = bench.stage_bytes(wl, 0.5)
+    assert bench.step_bytes(wl, 0.5)[1] == 312
+    assert sb["score"] == 2 * 2 * 128 * 64 * 2 + 2 * 4 * 18 * 64 * 2 + 1600
+    assert sb["budget"] == 16
+    assert sb["select"] == 1600 + 4 * 312 + 40
+    assert sb["compact"] == 4 * 312 * 64 * 2 + 4 * 312
+    assert sb["tail"] == 1600 + 4 * 312 * 64 * 2 + 4 * 312 + 40
