@@ -263,3 +263,42 @@ def test_prefill_and_given_statistics_validation(lib):
     assert evict_stats(ref(d), stats=P(0)) == 1
     assert b"row_stats" in lib.tgvkv_last_error()
     assert evict_stats(ref(d), ratio=1.5) == 1
+
+
+def test_binding_host_side(lib):
+    """The Python binding's host-only parts: descriptors from workloads and
+    options, output shapes and dtypes as the header states them (on the meta
+    device: no memory, no GPU), the retained-row capacity, errors raised."""
+    import torch
+    from paper_2606_03075_gb300 import api
+    wl = synth.WORKLOADS["qwen25"]
+    d = api.desc_for_workload(wl)
+    assert (d.L, d.H_q, d.H_kv, d.d, d.N, d.N_v, d.n_win) == (
+        wl.L, wl.H_q, wl.H_kv, wl.d, wl.N, wl.N_v, wl.n_win)
+    assert d.w_layer_stride == wl.n_win and d.softmax_scale == 0.0
+    assert (d.budget_basis, d.weight_mode, d.keep_first, d.keep_last, d.budget_stat,
+            d.head_budgets) == (0, 0, 0, 0, 0, 0)
+    o = api.desc_for_workload(wl, 0.125, basis="all", weights="eq7", keep_first=4, keep_last=1,
+                              stat="uniform", head_budgets=True, w_layer_stride=0)
+    assert (o.budget_basis, o.weight_mode, o.keep_first, o.keep_last, o.budget_stat,
+            o.head_budgets, o.w_layer_stride) == (1, 1, 4, 1, 2, 1, 0)
+    assert o.softmax_scale == 0.125
+    assert api.budget_units(d) == wl.L and api.budget_units(o) == wl.L * wl.H_kv
+    r = 0.05
+    rows = wl.H_kv * (wl.L * wl.N_t + oracle.vision_budget_total(r, wl.N_v, wl.L))
+    assert api.tgvkv_retained_rows(d, r) == rows
+    out = api.alloc_outputs(d, r, device="meta")
+    assert tuple(out.scores.shape) == (wl.L, wl.H_kv, wl.N_v) and out.scores.dtype == torch.float32
+    assert tuple(out.tvb_stat.shape) == (wl.L,) and out.budgets.dtype == torch.int32
+    assert tuple(out.offsets.shape) == (wl.L * wl.H_kv + 1,) and out.offsets.dtype == torch.int64
+    assert tuple(out.idx.shape) == (rows,) and out.idx.dtype == torch.int32
+    assert tuple(out.k_out.shape) == (rows, wl.d) == tuple(out.v_out.shape)
+    assert out.k_out.dtype == torch.bfloat16
+    heads = api.alloc_outputs(api.desc_for_workload(wl, head_budgets=True), r, device="meta")
+    assert tuple(heads.budgets.shape) == (wl.L * wl.H_kv,) == tuple(heads.tvb_stat.shape)
+    with pytest.raises(api.TgvkvError):
+        api.tgvkv_retained_rows(d, 1.5)
+    with pytest.raises(api.TgvkvError):
+        api.tgvkv_workspace_size(api.make_desc(1, 2, 2, 96, 10, 5, 2))
+    with pytest.raises(KeyError):
+        api.make_desc(1, 2, 2, 64, 10, 5, 2, basis="text")
