@@ -179,7 +179,7 @@ def main(pytest_args, src=SRC, funcs=None):
     try:
         for d in ("tests", "oracle", "paper_2606_03075_gb300", "profiles"):
             shutil.copytree(os.path.join(REPO, d), os.path.join(work, d),
-                            ignore=shutil.ignore_patterns("*.so", "__pycache__", "_build*"))
+                            ignore=shutil.ignore_patterns("__pycache__", "_build*"))
         for f in ("pytest.ini", "bench.py"):
             shutil.copy(os.path.join(REPO, f), work)
         base = ast.parse(open(os.path.join(REPO, src)).read())
