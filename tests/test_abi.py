@@ -101,6 +101,23 @@ def test_descriptor_limits(lib):
     assert ws(n_win=0) > 0 and ws(N_v=0) > 0 and ws(N_v=100) > 0
 
 
+def test_descriptor_edges_accepted_and_bad_scales_rejected(lib):
+    """The smallest valid shapes, a shared weight row and a cache of more than
+    2^30 key rows pass validation; a negative weight stride and a softmax scale
+    that is not finite are rejected (a scale <= 0 means 1/sqrt(d))."""
+    def ws(**kw):
+        return lib.tgvkv_workspace_size(ctypes.byref(_desc(**kw)))
+
+    assert ws(H_q=1, H_kv=1) > 0
+    assert ws(N=1, N_v=0) > 0 and ws(N=1, N_v=1) > 0
+    assert ws(w_layer_stride=0) > 0
+    assert ws(w_layer_stride=-1) == 0
+    assert ws(L=255, H_q=257, H_kv=257, N=32768, N_v=100) > 0   # 2147450880 K rows
+    for bad in (float("nan"), float("inf"), float("-inf")):
+        assert ws(softmax_scale=bad) == 0, bad
+    assert ws(softmax_scale=-1.0) > 0 and ws(softmax_scale=0.0) > 0
+
+
 def test_host_budget_arithmetic_matches_oracle(lib):
     ref = ctypes.byref
     for name, wl in synth.WORKLOADS.items():
