@@ -113,6 +113,7 @@ def test_descriptor_edges_accepted_and_bad_scales_rejected(lib):
     assert ws(w_layer_stride=0) > 0
     assert ws(w_layer_stride=-1) == 0
     assert ws(L=255, H_q=257, H_kv=257, N=32768, N_v=100) > 0   # 2147450880 K rows
+    assert ws(L=255, H_q=257, H_kv=257, n_win=32768, w_layer_stride=32768) > 0   # Q rows alike
     for bad in (float("nan"), float("inf"), float("-inf")):
         assert ws(softmax_scale=bad) == 0, bad
     assert ws(softmax_scale=-1.0) > 0 and ws(softmax_scale=0.0) > 0
